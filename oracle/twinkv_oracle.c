@@ -1,0 +1,324 @@
+/*
+ * twinkv_oracle.c -- reference oracle for the TwinKV redundancy audit and repair pass
+ * (arXiv 2608.27128).
+ *
+ * TEST INFRASTRUCTURE ONLY.  This file is a plain, slow, obviously-correct CPU
+ * restatement of the paper's definitions, in fp64.  Only the test suite, the smoke
+ * check of __graft_entry__ and the cpu_baseline leg of bench.py may load it.  The
+ * CUDA library never links, includes or calls it, and it shares no code with the
+ * CUDA library.
+ *
+ * What it computes, by paper passage:
+ *   Sec. 3.2, Eq. 1      sim(i,j) = khat_i . khat_j with khat_i = k_i / ||k_i||_2
+ *   Sec. 3.2, twin rule  j is a twin candidate of i only if |i-j| > w (and j != i)
+ *   Sec. 3.4, Eq. 4      b_i(S0) = max over j in S0, |i-j| > w, j != i of sim(i,j);
+ *                        -1 when no such j exists
+ *   (b_all)              the same maximum over every j (the twin relation of Sec. 3.2)
+ *   Sec. 3.4, orphan     i not in S0 and b_i(S0) < tau
+ *   Sec. 3.4, donor      j in S0, outside the sink/recent regions (Sec. 3.2, protected
+ *                        regions), and b_j(S0) >= tau
+ *   Sec. 3.4, repair     rank orphans by ascending b, donors by descending b,
+ *                        m = min(|O|,|D|), evict the m most severe donors and admit
+ *                        the m most severe orphans; |S1| = |S0|
+ *
+ * Readings where the paper is silent (each one is listed in the design notes):
+ *   - a key with zero norm has khat = 0, so its similarity with every key is 0;
+ *   - equal similarities: the lower position j wins the argmax;
+ *   - equal severities: the lower position comes first, for orphans and donors;
+ *   - the k-th most severe donor is paired with the k-th most severe orphan;
+ *   - b is computed once on S0; nothing is recomputed after a swap;
+ *   - threshold comparisons use the threshold rounded to float, widened to double,
+ *     so that a float implementation and this oracle compare against the same number;
+ *   - keys are bf16 bit patterns; float32 keys are first rounded to bf16,
+ *     round-to-nearest-even.
+ *
+ * Parity pins for every function here live in tests/test_oracle_pins.py and
+ * tests/golden/ (closed forms, hand-derived worked examples, a float64 numpy matmul,
+ * brute-force ranking and the paper's invariants).
+ */
+#include <math.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+
+/* ---- bf16 helpers (input decoding only) ---------------------------------------- */
+
+/* bf16 is the upper half of an IEEE binary32: decoding is exact. */
+static double bf16_to_double(uint16_t h)
+{
+    uint32_t bits = ((uint32_t)h) << 16;
+    float f;
+    memcpy(&f, &bits, sizeof f);
+    return (double)f;
+}
+
+/* float32 -> bf16, round to nearest, ties to even (finite inputs). */
+void twk_oracle_round_bf16(const float* in, uint16_t* out, long n)
+{
+    for (long t = 0; t < n; ++t) {
+        uint32_t bits;
+        memcpy(&bits, &in[t], sizeof bits);
+        uint32_t lower = bits & 0xFFFFu;
+        uint32_t upper = bits >> 16;
+        if (lower > 0x8000u || (lower == 0x8000u && (upper & 1u)))
+            upper += 1u;
+        out[t] = (uint16_t)upper;
+    }
+}
+
+/* ---- Eq. 1 ------------------------------------------------------------------------ */
+
+/* khat = k / ||k||_2 for every key of one (layer, head); zero keys stay zero. */
+static void normalise_keys(const uint16_t* keys, int N, int d, double* khat)
+{
+    for (int i = 0; i < N; ++i) {
+        double sq = 0.0;
+        for (int t = 0; t < d; ++t) {
+            double v = bf16_to_double(keys[(long)i * d + t]);
+            sq += v * v;
+        }
+        double norm = sqrt(sq);
+        for (int t = 0; t < d; ++t) {
+            double v = bf16_to_double(keys[(long)i * d + t]);
+            khat[(long)i * d + t] = (norm > 0.0) ? v / norm : 0.0;
+        }
+    }
+}
+
+static double dot(const double* a, const double* b, int d)
+{
+    double s = 0.0;
+    for (int t = 0; t < d; ++t)
+        s += a[t] * b[t];
+    return s;
+}
+
+/* sim(i, j) of Eq. 1 for keys i and j of one (layer, head) stored as bf16 rows of
+ * length d.  Used by the comparator to score a candidate twin. */
+double twk_oracle_sim(const uint16_t* key_i, const uint16_t* key_j, int d)
+{
+    double ni = 0.0, nj = 0.0;
+    for (int t = 0; t < d; ++t) {
+        double a = bf16_to_double(key_i[t]), b = bf16_to_double(key_j[t]);
+        ni += a * a;
+        nj += b * b;
+    }
+    ni = sqrt(ni);
+    nj = sqrt(nj);
+    double s = 0.0;
+    for (int t = 0; t < d; ++t) {
+        double a = (ni > 0.0) ? bf16_to_double(key_i[t]) / ni : 0.0;
+        double b = (nj > 0.0) ? bf16_to_double(key_j[t]) / nj : 0.0;
+        s += a * b;
+    }
+    return s;
+}
+
+/* ---- Eq. 4 and the best twin over all keys ------------------------------------- */
+
+/*
+ * For each unit u (one layer and KV head) and each requested row i, scan every
+ * position j in increasing order and keep
+ *   b_all / t_all : the largest sim(i,j) over j with |i-j| > w (j != i follows from
+ *                   w >= 0) and its position (first maximum wins, so the lowest j);
+ *   b_ret / t_ret : the same restricted to j with mask[j] != 0 (Eq. 4);
+ *   b_all2/b_ret2 : the second-largest value of each scan (the largest value over
+ *                   the eligible j other than the argmax), -INFINITY if there is none.
+ * An empty candidate set gives b = -1 and t = -1 (Eq. 4).
+ *
+ * keys  : bf16 bits [U][N][d]
+ * mask  : [U][N] (0 = evicted, non-zero = retained) or NULL (then b_ret/t_ret/b_ret2
+ *         are not written)
+ * rows  : list of nrows row positions evaluated in every unit, or NULL for all N rows
+ * out   : [U][nrows]
+ * Rows are independent; OpenMP (when compiled in) splits them across threads.
+ */
+void twk_oracle_audit(const uint16_t* keys, int U, int N, int d, const uint8_t* mask,
+                      int window, const int32_t* rows, int nrows, double* b_all,
+                      int32_t* t_all, double* b_all2, double* b_ret, int32_t* t_ret,
+                      double* b_ret2)
+{
+    if (rows == NULL)
+        nrows = N;
+    double* khat = (double*)malloc(sizeof(double) * (size_t)N * (size_t)d);
+    for (int u = 0; u < U; ++u) {
+        const uint16_t* K = keys + (long)u * N * d;
+        const uint8_t* S0 = mask ? mask + (long)u * N : NULL;
+        normalise_keys(K, N, d, khat);
+#pragma omp parallel for schedule(dynamic, 8)
+        for (int r = 0; r < nrows; ++r) {
+            int i = rows ? rows[r] : r;
+            double best = -1.0, second = -INFINITY;
+            int arg = -1;
+            double rbest = -1.0, rsecond = -INFINITY;
+            int rarg = -1;
+            for (int j = 0; j < N; ++j) {
+                int dist = (i > j) ? i - j : j - i;
+                if (j == i || dist <= window)
+                    continue;
+                double s = dot(&khat[(long)i * d], &khat[(long)j * d], d);
+                if (arg < 0 || s > best) {
+                    if (arg >= 0)
+                        second = best;
+                    best = s;
+                    arg = j;
+                } else if (s > second) {
+                    second = s;
+                }
+                if (S0 && S0[j]) {
+                    if (rarg < 0 || s > rbest) {
+                        if (rarg >= 0)
+                            rsecond = rbest;
+                        rbest = s;
+                        rarg = j;
+                    } else if (s > rsecond) {
+                        rsecond = s;
+                    }
+                }
+            }
+            long o = (long)u * nrows + r;
+            b_all[o] = best;
+            t_all[o] = arg;
+            if (b_all2)
+                b_all2[o] = second;
+            if (S0) {
+                b_ret[o] = rbest;
+                t_ret[o] = rarg;
+                if (b_ret2)
+                    b_ret2[o] = rsecond;
+            }
+        }
+    }
+    free(khat);
+}
+
+/* ---- Sec. 3.4: orphans, donors, severity ranking and the swap ------------------ */
+
+typedef struct {
+    double b;
+    int32_t pos;
+} ranked;
+
+/* orphans: ascending b, then ascending position */
+static int cmp_orphan(const void* pa, const void* pb)
+{
+    const ranked* a = (const ranked*)pa;
+    const ranked* b = (const ranked*)pb;
+    if (a->b < b->b) return -1;
+    if (a->b > b->b) return 1;
+    return (a->pos > b->pos) - (a->pos < b->pos);
+}
+
+/* donors: descending b, then ascending position */
+static int cmp_donor(const void* pa, const void* pb)
+{
+    const ranked* a = (const ranked*)pa;
+    const ranked* b = (const ranked*)pb;
+    if (a->b > b->b) return -1;
+    if (a->b < b->b) return 1;
+    return (a->pos > b->pos) - (a->pos < b->pos);
+}
+
+/*
+ * One unit of the repair pass.  b[N] = b_i(S0) (Eq. 4), mask[N] = S0 (values 0/1),
+ * tau = the threshold (already rounded to float and widened by the caller).
+ * Protected: i < n_sink or i >= N - n_recent.
+ * Writes out_mask[N] = S1, swaps[2k] = evicted donor, swaps[2k+1] = admitted orphan
+ * for k < m, and the orphan/donor flags (either may be NULL).  Returns m.
+ */
+static int repair_unit(int N, const double* b, const uint8_t* mask, double tau, int n_sink,
+                       int n_recent, uint8_t* out_mask, int32_t* swaps, uint8_t* is_orphan,
+                       uint8_t* is_donor)
+{
+    ranked* orphans = (ranked*)malloc(sizeof(ranked) * (size_t)(N > 0 ? N : 1));
+    ranked* donors = (ranked*)malloc(sizeof(ranked) * (size_t)(N > 0 ? N : 1));
+    int n_orphans = 0, n_donors = 0;
+    for (int i = 0; i < N; ++i) {
+        int retained = mask[i] != 0;
+        int protected_pos = (i < n_sink) || (i >= N - n_recent);
+        int orphan = !retained && (b[i] < tau);
+        int donor = retained && !protected_pos && (b[i] >= tau);
+        if (orphan) {
+            orphans[n_orphans].b = b[i];
+            orphans[n_orphans].pos = i;
+            ++n_orphans;
+        }
+        if (donor) {
+            donors[n_donors].b = b[i];
+            donors[n_donors].pos = i;
+            ++n_donors;
+        }
+        if (is_orphan) is_orphan[i] = (uint8_t)orphan;
+        if (is_donor) is_donor[i] = (uint8_t)donor;
+    }
+    qsort(orphans, (size_t)n_orphans, sizeof(ranked), cmp_orphan);
+    qsort(donors, (size_t)n_donors, sizeof(ranked), cmp_donor);
+    int m = n_orphans < n_donors ? n_orphans : n_donors;
+    for (int i = 0; i < N; ++i)
+        out_mask[i] = mask[i];
+    for (int k = 0; k < m; ++k) {
+        out_mask[donors[k].pos] = 0;
+        out_mask[orphans[k].pos] = 1;
+        swaps[2 * k] = donors[k].pos;
+        swaps[2 * k + 1] = orphans[k].pos;
+    }
+    free(orphans);
+    free(donors);
+    return m;
+}
+
+/*
+ * Repair over U units.  b[U][N] in double; budget[U] (or NULL = no check); the
+ * per-unit swap list has room for N/2 pairs (m <= min(K, N-K) <= N/2), so
+ * swaps is [U][N/2][2].  status[u]: 0 ok, 1 mask value outside {0,1}, 3 popcount of
+ * the mask differs from budget[u]; a failed unit gets nswaps = -1 and S1 = S0.
+ */
+void twk_oracle_repair(int U, int N, const double* b, const uint8_t* mask,
+                       const int32_t* budget, float threshold, int n_sink, int n_recent,
+                       uint8_t* out_mask, int32_t* swaps, int32_t* nswaps, int32_t* status,
+                       uint8_t* is_orphan, uint8_t* is_donor)
+{
+    double tau = (double)threshold;
+    long cap = 2L * (N / 2);
+    for (int u = 0; u < U; ++u) {
+        const uint8_t* S0 = mask + (long)u * N;
+        int bad_value = 0, count = 0;
+        for (int i = 0; i < N; ++i) {
+            if (S0[i] > 1) bad_value = 1;
+            count += S0[i] != 0;
+        }
+        int st = 0;
+        if (bad_value)
+            st = 1;
+        else if (budget && budget[u] != count)
+            st = 3;
+        status[u] = st;
+        if (st != 0) {
+            memcpy(out_mask + (long)u * N, S0, (size_t)N);
+            nswaps[u] = -1;
+            if (is_orphan) memset(is_orphan + (long)u * N, 0, (size_t)N);
+            if (is_donor) memset(is_donor + (long)u * N, 0, (size_t)N);
+            continue;
+        }
+        nswaps[u] = repair_unit(N, b + (long)u * N, S0, tau, n_sink, n_recent,
+                                out_mask + (long)u * N, swaps + (long)u * cap,
+                                is_orphan ? is_orphan + (long)u * N : NULL,
+                                is_donor ? is_donor + (long)u * N : NULL);
+    }
+}
+
+/* Selection-only entry: the same repair on float32 b values (for example, a GPU's own
+ * b), widened exactly to double, so every comparison equals the float comparison. */
+void twk_oracle_repair_f32(int U, int N, const float* b, const uint8_t* mask,
+                           const int32_t* budget, float threshold, int n_sink, int n_recent,
+                           uint8_t* out_mask, int32_t* swaps, int32_t* nswaps,
+                           int32_t* status, uint8_t* is_orphan, uint8_t* is_donor)
+{
+    long n = (long)U * N;
+    double* bd = (double*)malloc(sizeof(double) * (size_t)(n > 0 ? n : 1));
+    for (long t = 0; t < n; ++t)
+        bd[t] = (double)b[t];
+    twk_oracle_repair(U, N, bd, mask, budget, threshold, n_sink, n_recent, out_mask, swaps,
+                      nswaps, status, is_orphan, is_donor);
+    free(bd);
+}
