@@ -1,0 +1,350 @@
+"""Throughput of the TwinKV audit + repair pass (arXiv 2608.27128) on one GB300.
+
+One step = one full pass over a prefilled KV cache of the Qwen3-4B shape
+(36 layers x 8 KV heads x 16384 keys x d=128, bf16, synthetic): 1/||k|| and the
+retained-first column gather, the fused similarity audit (b_i(all) and b_i(S0) with
+their argmaxes, Sec. 3.2 Eq. 1 and Sec. 3.4 Eq. 4) and the orphan/donor swap
+(Sec. 3.4), all through the C ABI call twinkv_repair.  Metric: audited keys/s =
+L*H*N / step time.  The keys (1.2 GB) exceed the 129 MB L2, so no flush is needed
+between steps.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+With torchrun (N > 1) every rank runs the same workload on its own GPU (independent
+replicas: weak scaling); the reported time is the maximum over ranks and the value is
+the keys all ranks processed divided by it.  ``--impl reference`` times the fp64 CPU
+oracle, on the host cores, on a bounded sample of the same workload.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "audited keys/sec (L×H×N) at Qwen3-4B shape; % tensor-core peak"
+PEAKS_FILE = os.path.join(ROOT, "MEASURED_PEAKS.json")
+FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+
+def peaks():
+    try:
+        with open(PEAKS_FILE) as f:
+            p = json.load(f)
+        return p, "measured"
+    except (OSError, ValueError):
+        return dict(FALLBACK), "fallback"
+
+
+def workload_config(w, ratio):
+    return {
+        "workload": f"Qwen3-4B KV cache {w.L}x{w.H}x{w.N}x{w.d} bf16 (synthetic), ratio {ratio}",
+        "L": w.L, "H": w.H, "N": w.N, "d": w.d, "ratio": ratio, "tau": w.tau,
+        "window": 32, "n_sink": 4, "n_recent": 64,
+        "budget_per_unit": None,
+        "l2": "inputs larger than L2 (keys 1.2 GB > 129 MB); no flush",
+        "parallelism": "replicas",
+    }
+
+
+class ClockSampler:
+    """nvidia-smi clock/throttle samples during the timed region."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = os.path.join(ROOT, "gpurun_out", f"clocks_gpu{gpu_index}.csv")
+
+    def __enter__(self):
+        try:
+            os.makedirs(os.path.dirname(self.path), exist_ok=True)
+            self.f = open(self.path, "w")
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=self.f, stderr=subprocess.DEVNULL)
+            time.sleep(0.3)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            time.sleep(0.15)
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+            self.f.close()
+
+    def summary(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        rows = []
+        with open(self.path) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) >= 9:
+                    rows.append(parts)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+        sm = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
+        mx = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[k] for r in rows for k in range(4) if r[5 + k] == "Active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None, "reasons": reasons,
+                "samples": len(rows),
+                "power_w_max": max((float(r[3]) for r in rows
+                                    if r[3].replace(".", "").isdigit()), default=None)}
+
+
+def dist_setup():
+    import torch
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    return world, rank, local
+
+
+def max_over_ranks(x: float, world: int) -> float:
+    if world == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def cpu_sample(w, ratio, units, rows_per_unit):
+    """Oracle (fp64, host cores) on `units` units, `rows_per_unit` rows each (all columns).
+
+    Returns (keys/s, seconds, threads, description)."""
+    import oracle
+    from paper_2608_27128_gb300 import synth
+    oracle.build()
+    ul = [(u // w.H, u % w.H) for u in range(units)]
+    keys, _ = synth.keys(w, units=ul)
+    S0 = synth.masks(w, ratio, units=ul)
+    rows = np.sort(np.random.default_rng(0).choice(w.N, size=rows_per_unit, replace=False))
+    t0 = time.perf_counter()
+    oracle.audit(keys, S0, window=32, rows=rows)
+    dt = time.perf_counter() - t0
+    threads = int(os.environ.get("OMP_NUM_THREADS", os.cpu_count() or 1))
+    n = units * rows_per_unit
+    desc = (f"{units} unit(s) x {rows_per_unit} rows (of {w.N}), every column, both maxima; "
+            "the O(N d) repair step is not in the sample")
+    return n / dt, dt, threads, desc
+
+
+def run_reference(args, w, ratio):
+    world, rank, _ = int(os.environ.get("WORLD_SIZE", "1")), int(os.environ.get("RANK", "0")), 0
+    if rank != 0:
+        return
+    vals = []
+    for _ in range(args.warmup + args.steps):
+        v, dt, threads, desc = cpu_sample(w, ratio, args.cpu_units, args.cpu_rows)
+        vals.append((v, dt))
+    timed = vals[args.warmup:]
+    v = statistics.median(x[0] for x in timed)
+    ms = statistics.median(x[1] for x in timed) * 1e3
+    line = {
+        "metric": METRIC, "value": v, "unit": "keys/s", "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic", "config": workload_config(w, ratio), "impl": "reference",
+        "cpu_baseline": {"value": v, "unit": "keys/s", "cores": threads, "kind": "oracle",
+                         "sample": desc},
+        "e2e": {"value": v, "unit": "keys/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def run_ours(args, w, ratio):
+    import torch
+
+    from paper_2608_27128_gb300 import synth
+    from paper_2608_27128_gb300 import twinkv as tk
+
+    world, rank, local = dist_setup()
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    tk.load()
+
+    keys_np, _ = synth.keys(w)
+    S0_np = synth.masks(w, ratio)
+    L, H, N, d = w.L, w.H, w.N, w.d
+    U = L * H
+    keys_h = torch.from_numpy(keys_np.view(np.int16).reshape(L, H, N, d)).view(torch.bfloat16)
+    mask_h = torch.from_numpy(S0_np.reshape(L, H, N))
+    budget_h = torch.from_numpy(S0_np.sum(1).astype(np.int32))
+    keys = keys_h.to(dev)
+    mask = mask_h.to(dev)
+    budget = budget_h.to(dev)
+    shape = tk.shape_of(keys)
+    ws = tk.workspace(shape, tk.OP_REPAIR, dev)
+    out = None
+
+    def step(k=keys, m=mask, b=budget):
+        nonlocal out
+        out = tk.twinkv_repair(k, m, b, threshold=w.tau, want_all=True, out=out, ws=ws)
+        return out
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    assert tk.twinkv_get_last_error() == tk.OK
+
+    # ---- device-resident timed region
+    stream = torch.cuda.current_stream()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    barrier(world)
+    with ClockSampler(local) as clocks:
+        torch.cuda.synchronize()
+        tk.twinkv_profile_begin()
+        e0.record(stream)
+        for _ in range(args.steps):
+            step()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        prof = tk.twinkv_profile_end()
+    barrier(world)
+    ms = max_over_ranks(e0.elapsed_time(e1) / args.steps, world)
+    assert tk.twinkv_get_last_error() == tk.OK
+    value = world * U * N / (ms * 1e-3)
+
+    # ---- end to end: pinned host inputs -> device, the call, results -> host
+    keys_p = keys_h.pin_memory()
+    mask_p = mask_h.pin_memory()
+    budget_p = budget_h.pin_memory()
+    S1_p = torch.empty((L, H, N), dtype=torch.uint8).pin_memory()
+    sw_p = torch.empty((U, N // 2, 2), dtype=torch.int32).pin_memory()
+    ns_p = torch.empty((U,), dtype=torch.int32).pin_memory()
+    kd = torch.empty_like(keys)
+    md = torch.empty_like(mask)
+    bd = torch.empty_like(budget)
+
+    def e2e_step():
+        kd.copy_(keys_p, non_blocking=True)
+        md.copy_(mask_p, non_blocking=True)
+        bd.copy_(budget_p, non_blocking=True)
+        o = step(kd, md, bd)
+        S1_p.copy_(o["mask"], non_blocking=True)
+        sw_p.copy_(o["swaps"], non_blocking=True)
+        ns_p.copy_(o["nswaps"], non_blocking=True)
+
+    for _ in range(2):
+        e2e_step()
+    torch.cuda.synchronize()
+    e2e_steps = max(3, args.steps // 2)
+    barrier(world)
+    f0, f1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    f0.record(stream)
+    for _ in range(e2e_steps):
+        e2e_step()
+    f1.record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = max_over_ranks(f0.elapsed_time(f1) / e2e_steps, world)
+    # the step's results match the device-resident run
+    assert torch.equal(S1_p, out["mask"].cpu())
+    h2d = keys_h.numel() * 2 + mask_h.numel() + budget_h.numel() * 4
+    d2h = S1_p.numel() + sw_p.numel() * 4 + ns_p.numel() * 4
+
+    if rank != 0:
+        return
+
+    # ---- roofline of the dominant kernel (the fused audit)
+    pk, pk_kind = peaks()
+    n_audit, audit_ms = prof["audit"]
+    audit_ms_per = audit_ms / max(n_audit, 1)
+    flops = 2.0 * N * N * d * U
+    achieved = flops / (audit_ms_per * 1e-3) / 1e12
+    peak = pk["bf16_tflops_sustained"]
+    launches = sum(n for n, _ in prof.values())
+    traffic = None
+    tfile = os.path.join(ROOT, "profiles", "audit_traffic.json")
+    if os.path.exists(tfile):
+        try:
+            with open(tfile) as f:
+                tinfo = json.load(f)
+            if tinfo.get("workload") == "qwen" and tinfo.get("kernel_rev") == KERNEL_REV:
+                traffic = tinfo.get("bytes_per_launch")
+        except (OSError, ValueError):
+            traffic = None
+
+    line = {
+        "metric": METRIC, "value": value, "unit": "keys/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic", "config": workload_config(w, ratio),
+        "tflops_audit": achieved,
+        "frac_of_burst_peak": achieved / pk["bf16_tflops"],
+        "roofline": {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+                     "frac": achieved / peak, "traffic": traffic,
+                     "peak_kind": f"{pk_kind} bf16_tflops_sustained (kernel timed inside a "
+                                  "long loop)",
+                     "kernel": "twk audit_kernel", "flops_per_launch": flops,
+                     "ms_per_launch": audit_ms_per},
+        "kernel_ms_per_step": {k: (t / max(n, 1)) for k, (n, t) in prof.items()},
+        "gpu_launches": launches,
+        "e2e": {"value": world * U * N / (e2e_ms * 1e-3), "unit": "keys/s",
+                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms},
+        "clocks": clocks.summary(),
+    }
+    if not args.no_cpu:
+        v, dt, threads, desc = cpu_sample(w, ratio, args.cpu_units, args.cpu_rows)
+        line["cpu_baseline"] = {"value": v, "unit": "keys/s", "cores": threads,
+                                "kind": "oracle", "sample": desc, "seconds": dt}
+    print(json.dumps(line), flush=True)
+
+
+# Revision of the audit kernel the committed DRAM-traffic capture refers to.
+KERNEL_REV = "v1"
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
+    ap.add_argument("--ratio", type=float, default=0.5)
+    ap.add_argument("--cpu-units", type=int, default=8)
+    ap.add_argument("--cpu-rows", type=int, default=16384)
+    ap.add_argument("--no-cpu", action="store_true")
+    args = ap.parse_args()
+    from paper_2608_27128_gb300 import synth
+    w = synth.get("qwen")
+    if args.impl == "reference":
+        run_reference(args, w, args.ratio)
+    else:
+        run_ours(args, w, args.ratio)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,218 @@
+/*
+ * twinkv.h -- C ABI of the GB300 (sm_103a) TwinKV key-redundancy audit and repair
+ * pass (arXiv 2608.27128, "TwinKV: A Composable Repair Pass for KV Cache Eviction via
+ * Pairwise Key Redundancy").
+ *
+ * Terms, after the paper:
+ *   unit        one (layer, KV head); the pass runs on every unit independently
+ *               (Sec. 3.1, problem setup).
+ *   keys        k_1..k_N of a unit, post-RoPE as stored in the cache (Sec. 3.2).
+ *   sim(i,j)    cosine similarity of keys i and j (Sec. 3.2, Eq. 1).
+ *   window w    positions with |i-j| <= w never count as twins (Sec. 3.2).
+ *   S0          the retained set a wrapped eviction policy produced, K = |S0|
+ *               (Sec. 3.4).
+ *   b_i(S0)     best surviving twin similarity: max of sim(i,j) over j in S0 with
+ *               |i-j| > w, or -1 if no such j (Sec. 3.4, Eq. 4).
+ *   b_i(all)    the same maximum over every position j.
+ *   orphan      i not in S0 with b_i(S0) < tau (Sec. 3.4).
+ *   donor       j in S0, outside the protected sink and recent regions (Sec. 3.2),
+ *               with b_j(S0) >= tau (Sec. 3.4).
+ *   repair      m = min(|orphans|, |donors|); evict the m donors of largest b,
+ *               admit the m orphans of smallest b; |S1| = |S0| (Sec. 3.4).
+ *
+ * Readings of points the paper leaves open, applied by every call:
+ *   - equal similarities: the lowest position j is the twin;
+ *   - equal severities: the lower position ranks first, for orphans and donors;
+ *   - the k-th donor (by severity) is paired with the k-th orphan in the swap list;
+ *   - b is computed once on S0; nothing is recomputed after a swap;
+ *   - a key of zero norm has similarity 0 with every key;
+ *   - float32 keys are rounded to bf16 (nearest, ties to even) before anything else.
+ *
+ * Memory.  Every pointer argument except `params` (host) is a DEVICE pointer owned by
+ * the caller.  The library allocates nothing: calls that need scratch memory take a
+ * caller-owned device `workspace` of at least twinkv_workspace_size() bytes (256-byte
+ * aligned).  Tensors are dense, row-major, innermost dimension last:
+ *   keys        [L][H][N][d]   bf16 (raw 16-bit patterns) or float32
+ *   masks       [L][H][N]      uint8, 0 = evicted, 1 = retained
+ *   scores      [L][H][N]      float32
+ *   twins       [L][H][N]      int32 position in 0..N-1, or -1
+ *   per-unit    [L*H]          int32
+ *   swaps       [L*H][N/2][2]  int32 pairs (evicted donor, admitted orphan); unit u's
+ *                              list starts at element u*2*(N/2); twinkv_swaps_capacity()
+ *                              gives the total element count
+ *
+ * Streams.  `stream` is a cudaStream_t passed as void* (NULL = legacy default stream).
+ * Every call only enqueues work on it and returns; outputs are valid once the stream
+ * has completed.
+ *
+ * Errors.  Argument errors that the host can see (null pointers, sizes, d, dtype,
+ * window, threshold, a too-small workspace) are returned at once and nothing is
+ * enqueued.  Per-unit data errors are found on the device and reported in
+ * out_status[u]: TWINKV_ERR_BUDGET when the popcount of the unit's mask differs from
+ * budget[u], TWINKV_ERR_INVALID_ARG when a mask byte is neither 0 nor 1; such a unit
+ * gets out_nswaps[u] = -1 and out_mask equal to its input mask.  A device-side wait
+ * that gives up (TWINKV_ERR_TIMEOUT) and asynchronous CUDA errors are reported by
+ * twinkv_get_last_error().  No call throws, traps or aborts the process.
+ *
+ * Limits: d in {64, 128}; 1 <= N <= 1048576; L*H*N*d < 2^31 elements per tensor
+ * coordinate; L*H*(N rounded up to 256, plus 256) < 2^31 rows.
+ */
+#ifndef TWINKV_H
+#define TWINKV_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define TWINKV_ABI_VERSION 1
+
+typedef enum {
+    TWINKV_OK = 0,
+    TWINKV_ERR_INVALID_ARG = 1,   /* a host-visible argument is wrong, or a mask byte > 1 */
+    TWINKV_ERR_UNSUPPORTED = 2,   /* valid request this build does not cover (d, device) */
+    TWINKV_ERR_BUDGET = 3,        /* popcount(mask of unit u) != budget[u] */
+    TWINKV_ERR_CUDA = 4,          /* a CUDA runtime/driver call failed */
+    TWINKV_ERR_TIMEOUT = 5,       /* a device-side wait gave up; outputs are undefined */
+    TWINKV_ERR_WORKSPACE = 6      /* workspace missing, misaligned or too small */
+} twinkv_status;
+
+typedef enum { TWINKV_BF16 = 0, TWINKV_F32 = 1 } twinkv_dtype;
+
+/* keys[L][H][N][d] of element type `dtype` (a twinkv_dtype value). */
+typedef struct {
+    int32_t L, H, N, d;
+    int32_t dtype;
+} twinkv_shape;
+
+/* Scorer parameters (Sec. 3.2): threshold tau, local window w, protected regions. */
+typedef struct {
+    float threshold;     /* tau; twinkv_repair's own `threshold` argument overrides it */
+    int32_t window;      /* w >= 0 */
+    int32_t n_sink;      /* positions i < n_sink are protected (never donors) */
+    int32_t n_recent;    /* positions i >= N - n_recent are protected */
+} twinkv_params;
+
+/* Operations, for twinkv_workspace_size(). */
+typedef enum {
+    TWINKV_OP_REDUNDANCY = 0,
+    TWINKV_OP_REPAIR = 1,
+    TWINKV_OP_REPAIR_SELECT = 2
+} twinkv_op;
+
+/* Kernels, for the profiling hooks. */
+typedef enum {
+    TWINKV_KERNEL_PREP = 0,      /* bf16 rounding, norms, retained-first column gather */
+    TWINKV_KERNEL_AUDIT = 1,     /* fused similarity + masked max/argmax (Eq. 1, Eq. 4) */
+    TWINKV_KERNEL_REPAIR = 2,    /* classify, rank, select and swap (Sec. 3.4) */
+    TWINKV_KERNEL_COUNT = 3
+} twinkv_kernel;
+
+/* Paper defaults: tau = 0.85, w = 32, 4 sink and 64 recent positions (Sec. 3.2). */
+twinkv_params twinkv_default_params(void);
+
+/* Number of int32 elements out_swaps must hold: L*H*(N/2)*2.  0 on a bad shape. */
+size_t twinkv_swaps_capacity(twinkv_shape s);
+
+/* Workspace bytes `op` needs for shape s (0 on a bad shape or op). */
+size_t twinkv_workspace_size(twinkv_shape s, int32_t op);
+
+/*
+ * Best twin of every key over all other keys (Sec. 3.2, Eq. 1 and the twin window;
+ * the maximum b_i(all) behind the redundancy count of Eq. 2: r_i > 0 iff
+ * b_i(all) > tau).
+ *   keys       [L][H][N][d] device, dtype per s.dtype
+ *   window     w >= 0
+ *   out_score  [L][H][N] float32: b_i(all), or -1 when no position lies beyond w
+ *   out_twin   [L][H][N] int32: its position (lowest on ties), or -1
+ */
+twinkv_status twinkv_redundancy(const void* keys, twinkv_shape s, int32_t window,
+                                float* out_score, int32_t* out_twin, void* workspace,
+                                size_t workspace_bytes, void* stream);
+
+/*
+ * Audit of a retained set and the budget-exact repair swap (Sec. 3.4, Eq. 4 and the
+ * orphan/donor rule), all units in one pass.
+ *   keys           [L][H][N][d] device
+ *   retained_mask  [L][H][N] uint8, S0
+ *   budget         [L*H] int32 expected |S0| per unit, or NULL (no check)
+ *   threshold      tau (finite); overrides params->threshold
+ *   params         host pointer, or NULL for twinkv_default_params(); its window,
+ *                  n_sink and n_recent are used
+ *   out_mask       [L][H][N] uint8: S1
+ *   out_swaps      [L*H][N/2][2] int32: (evicted donor, admitted orphan), most severe
+ *                  first; entries past out_nswaps[u] are left untouched
+ *   out_nswaps     [L*H] int32: m, or -1 for a unit with a data error
+ *   out_score_ret  [L][H][N] float32 b_i(S0), or NULL
+ *   out_twin_ret   [L][H][N] int32 argmax of b_i(S0), or NULL
+ *   out_score_all  [L][H][N] float32 b_i(all), or NULL; when both this and
+ *                  out_twin_all are NULL the evicted columns are skipped entirely
+ *                  (O(N K d) instead of O(N^2 d), Sec. 3.5)
+ *   out_twin_all   [L][H][N] int32, or NULL
+ *   out_status     [L*H] int32 per-unit twinkv_status, or NULL
+ */
+twinkv_status twinkv_repair(const void* keys, twinkv_shape s, const uint8_t* retained_mask,
+                            const int32_t* budget, float threshold,
+                            const twinkv_params* params, uint8_t* out_mask,
+                            int32_t* out_swaps, int32_t* out_nswaps, float* out_score_ret,
+                            int32_t* out_twin_ret, float* out_score_all,
+                            int32_t* out_twin_all, int32_t* out_status, void* workspace,
+                            size_t workspace_bytes, void* stream);
+
+/*
+ * The classification, ranking and swap of twinkv_repair alone, on caller-supplied
+ * b_i(S0) values (Sec. 3.4).  Same arguments and outputs as twinkv_repair; s.d and
+ * s.dtype are ignored.  score_ret [L][H][N] float32 device.
+ */
+twinkv_status twinkv_repair_select(const float* score_ret, twinkv_shape s,
+                                   const uint8_t* retained_mask, const int32_t* budget,
+                                   float threshold, const twinkv_params* params,
+                                   uint8_t* out_mask, int32_t* out_swaps,
+                                   int32_t* out_nswaps, int32_t* out_status,
+                                   void* workspace, size_t workspace_bytes, void* stream);
+
+/* Static description of a status code. */
+const char* twinkv_status_string(twinkv_status st);
+
+/*
+ * Sticky asynchronous error of the current device: synchronizes the device, returns
+ * TWINKV_ERR_TIMEOUT if a kernel's wait gave up, TWINKV_ERR_CUDA on a pending CUDA
+ * error, else TWINKV_OK, and clears the sticky timeout.
+ */
+twinkv_status twinkv_get_last_error(void);
+
+/*
+ * Upper bound, in nanoseconds, on any single device-side wait of the kernels launched
+ * afterwards (default 2e9).  A wait that exceeds it makes the kernel record
+ * TWINKV_ERR_TIMEOUT, release its resources and return.
+ */
+twinkv_status twinkv_set_wait_timeout_ns(uint64_t ns);
+
+/*
+ * Exercises that give-up path: launches one block that takes tensor memory, waits on
+ * a barrier nothing will ever complete (bounded by timeout_ns), frees the tensor
+ * memory and returns.  Synchronizes the stream and writes the status the kernel
+ * recorded (TWINKV_ERR_TIMEOUT expected) to *out (host pointer).
+ */
+twinkv_status twinkv_wait_probe(uint64_t timeout_ns, int32_t* out, void* stream);
+
+/*
+ * Profiling hooks.  Between twinkv_profile_begin() and twinkv_profile_end(), every
+ * kernel launch of this library is bracketed by CUDA events on its stream.
+ * twinkv_profile_end() synchronizes those events and returns, per twinkv_kernel, the
+ * number of launches and their summed device time in milliseconds (arrays of
+ * TWINKV_KERNEL_COUNT host elements).
+ */
+twinkv_status twinkv_profile_begin(void);
+twinkv_status twinkv_profile_end(int32_t* launches, double* total_ms);
+
+/* Library build info: ABI version. */
+int32_t twinkv_abi_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* TWINKV_H */

@@ -1,0 +1,518 @@
+// twk_api.cu -- the C ABI of libtwinkv (declared in include/twinkv.h): argument
+// validation, workspace carving, TMA tensor maps and the launch sequence of the
+// TwinKV audit and repair pass (arXiv 2608.27128, Sec. 3.2 and 3.4).
+#include <cmath>
+#include <cstring>
+#include <mutex>
+#include <vector>
+
+#include "twinkv.h"
+#include "twk_internal.h"
+
+namespace twk {
+namespace {
+
+__device__ int g_error_word[4];   // sticky device-side status (see twk_ptx.cuh)
+__device__ int g_probe_word[4];   // status written by the wait probe
+
+constexpr int kMaxDevices = 64;
+constexpr int64_t kMaxN = 1 << 20;
+
+std::mutex g_mu;
+unsigned long long g_timeout_ns = 2000000000ull;
+
+struct DeviceInfo {
+    bool ready = false;
+    int sms = 0;
+    int cc_major = 0, cc_minor = 0;
+    int* err = nullptr;
+    int* probe = nullptr;
+};
+DeviceInfo g_dev[kMaxDevices];
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                  const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                  const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+EncodeTiledFn g_encode = nullptr;
+
+// ---------------------------------------------------------------- profiling hooks
+struct ProfRecord {
+    int kernel;
+    cudaEvent_t start, stop;
+};
+bool g_prof_on = false;
+std::vector<ProfRecord> g_prof;
+
+struct ProfScope {
+    int kernel;
+    cudaStream_t st;
+    cudaEvent_t start = nullptr, stop = nullptr;
+    ProfScope(int k, cudaStream_t s) : kernel(k), st(s)
+    {
+        if (!g_prof_on) return;
+        cudaEventCreate(&start);
+        cudaEventCreate(&stop);
+        cudaEventRecord(start, st);
+    }
+    ~ProfScope()
+    {
+        if (!start) return;
+        cudaEventRecord(stop, st);
+        std::lock_guard<std::mutex> lk(g_mu);
+        g_prof.push_back({kernel, start, stop});
+    }
+};
+
+twinkv_status cuda_status(cudaError_t e) { return e == cudaSuccess ? TWINKV_OK : TWINKV_ERR_CUDA; }
+
+// Current device's cached facts; sets them up on first use (outside stream capture).
+twinkv_status device_info(DeviceInfo** out)
+{
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices)
+        return TWINKV_ERR_CUDA;
+    std::lock_guard<std::mutex> lk(g_mu);
+    DeviceInfo& d = g_dev[dev];
+    if (!d.ready) {
+        if (cudaDeviceGetAttribute(&d.sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
+            cudaDeviceGetAttribute(&d.cc_major, cudaDevAttrComputeCapabilityMajor, dev) !=
+                cudaSuccess ||
+            cudaDeviceGetAttribute(&d.cc_minor, cudaDevAttrComputeCapabilityMinor, dev) !=
+                cudaSuccess)
+            return TWINKV_ERR_CUDA;
+        if (cudaGetSymbolAddress(reinterpret_cast<void**>(&d.err), g_error_word) != cudaSuccess ||
+            cudaGetSymbolAddress(reinterpret_cast<void**>(&d.probe), g_probe_word) !=
+                cudaSuccess)
+            return TWINKV_ERR_CUDA;
+        if (!g_encode) {
+            cudaDriverEntryPointQueryResult q;
+            void* fn = nullptr;
+            if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000,
+                                                 cudaEnableDefault, &q) != cudaSuccess ||
+                q != cudaDriverEntryPointSuccess || !fn)
+                return TWINKV_ERR_CUDA;
+            g_encode = reinterpret_cast<EncodeTiledFn>(fn);
+        }
+        d.ready = true;
+    }
+    // The kernels are built for sm_103a only.
+    if (d.cc_major != 10 || d.cc_minor != 3) return TWINKV_ERR_UNSUPPORTED;
+    *out = &d;
+    return TWINKV_OK;
+}
+
+// bf16 rows of length d: a 2-D tensor map [rows][d] with 128-byte swizzle and a box of
+// 64 elements x box_rows rows.
+twinkv_status make_map(CUtensorMap* map, const void* base, int64_t rows, int d, int box_rows)
+{
+    cuuint64_t dims[2] = {static_cast<cuuint64_t>(d), static_cast<cuuint64_t>(rows)};
+    cuuint64_t strides[1] = {static_cast<cuuint64_t>(d) * 2};
+    cuuint32_t box[2] = {64, static_cast<cuuint32_t>(box_rows)};
+    cuuint32_t estr[2] = {1, 1};
+    const CUresult r = g_encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base),
+                                dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                                CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS ? TWINKV_OK : TWINKV_ERR_CUDA;
+}
+
+// ---------------------------------------------------------------- shapes, workspace
+bool shape_ok(const twinkv_shape& s, bool need_d)
+{
+    if (s.L < 1 || s.H < 1 || s.N < 1 || s.N > kMaxN) return false;
+    const int64_t U = static_cast<int64_t>(s.L) * s.H;
+    if (U > (1 << 24)) return false;
+    if (!need_d) return U * s.N < (1LL << 31);
+    if (s.d != 64 && s.d != 128) return false;
+    if (s.dtype != TWINKV_BF16 && s.dtype != TWINKV_F32) return false;
+    if (U * s.N * s.d >= (1LL << 31)) return false;          // element offsets
+    if (U * column_stride(s.N) >= (1LL << 31)) return false; // TMA row coordinates
+    return true;
+}
+
+size_t up256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
+
+struct Layout {
+    size_t keys16 = 0, colrinv = 0, colpos = 0, kp = 0, rowrinv = 0, cnt = 0, kb = 0,
+           bret = 0, k0 = 0, i0 = 0, k1 = 0, i1 = 0;
+    size_t total = 0;
+};
+
+Layout layout(const twinkv_shape& s, int op)
+{
+    Layout L;
+    size_t off = 0;
+    auto take = [&](size_t bytes) {
+        const size_t o = off;
+        off += up256(bytes);
+        return o;
+    };
+    const size_t U = static_cast<size_t>(s.L) * s.H;
+    const size_t N = static_cast<size_t>(s.N);
+    if (op == TWINKV_OP_REDUNDANCY || op == TWINKV_OP_REPAIR) {
+        const size_t NP = static_cast<size_t>(column_stride(s.N));
+        if (s.dtype == TWINKV_F32) L.keys16 = take(U * N * s.d * 2);
+        L.colrinv = take(U * NP * 4);
+        L.colpos = take(U * NP * 4);
+        if (op == TWINKV_OP_REPAIR) {
+            L.kp = take(U * NP * s.d * 2);
+            L.rowrinv = take(U * N * 4);
+            L.cnt = take(U * N * 4);
+            L.kb = take(U * 4);
+            L.bret = take(U * N * 4);
+        }
+    }
+    if (op == TWINKV_OP_REPAIR || op == TWINKV_OP_REPAIR_SELECT) {
+        L.k0 = take(U * N * 4);
+        L.i0 = take(U * N * 4);
+        L.k1 = take(U * N * 4);
+        L.i1 = take(U * N * 4);
+    }
+    L.total = off;
+    return L;
+}
+
+template <typename T>
+T* at(void* ws, size_t off)
+{
+    return reinterpret_cast<T*>(static_cast<char*>(ws) + off);
+}
+
+twinkv_status check_ws(const twinkv_shape& s, int op, void* ws, size_t bytes, Layout* out)
+{
+    *out = layout(s, op);
+    if (out->total == 0) return TWINKV_OK;
+    if (!ws || (reinterpret_cast<uintptr_t>(ws) & 255) != 0 || bytes < out->total)
+        return TWINKV_ERR_WORKSPACE;
+    return TWINKV_OK;
+}
+
+// bf16 view of the keys (rounding float32 keys into the workspace first).
+twinkv_status keys_bf16(const void* keys, const twinkv_shape& s, void* ws, const Layout& L,
+                        cudaStream_t st, const uint16_t** out)
+{
+    if (s.dtype == TWINKV_BF16) {
+        *out = static_cast<const uint16_t*>(keys);
+        return TWINKV_OK;
+    }
+    uint16_t* k16 = at<uint16_t>(ws, L.keys16);
+    ProfScope p(TWINKV_KERNEL_PREP, st);
+    const int64_t n = static_cast<int64_t>(s.L) * s.H * s.N * s.d;
+    const cudaError_t e = launch_round_bf16(static_cast<const float*>(keys), k16, n, st);
+    *out = k16;
+    return cuda_status(e);
+}
+
+twinkv_status run_audit(const DeviceInfo& dev, const twinkv_shape& s, const uint16_t* keys16,
+                        const void* bkeys, int64_t b_rows, AuditArgs a, cudaStream_t st)
+{
+    CUtensorMap tmA, tmB;
+    const int64_t U = static_cast<int64_t>(s.L) * s.H;
+    twinkv_status r = make_map(&tmA, keys16, U * s.N, s.d, kBM);
+    if (r != TWINKV_OK) return r;
+    r = make_map(&tmB, bkeys, b_rows, s.d, kBN);
+    if (r != TWINKV_OK) return r;
+    const int64_t items = U * a.RB;
+    const int grid = static_cast<int>(items < dev.sms ? items : dev.sms);
+    ProfScope p(TWINKV_KERNEL_AUDIT, st);
+    return cuda_status(launch_audit(s.d, tmA, tmB, a, grid, st));
+}
+
+twinkv_status params_ok(const twinkv_params& p, float threshold)
+{
+    if (!std::isfinite(threshold)) return TWINKV_ERR_INVALID_ARG;
+    if (p.window < 0 || p.n_sink < 0 || p.n_recent < 0) return TWINKV_ERR_INVALID_ARG;
+    return TWINKV_OK;
+}
+
+twinkv_status launch_select(const twinkv_shape& s, const float* b, const uint8_t* mask,
+                            const int32_t* budget, float threshold, const twinkv_params& p,
+                            uint8_t* out_mask, int32_t* out_swaps, int32_t* out_nswaps,
+                            int32_t* out_status, void* ws, const Layout& L, cudaStream_t st)
+{
+    RepairArgs r;
+    r.U = s.L * s.H;
+    r.N = s.N;
+    r.b = b;
+    r.mask = mask;
+    r.budget = budget;
+    r.tau = threshold;
+    r.n_sink = p.n_sink;
+    r.n_recent = p.n_recent;
+    r.out_mask = out_mask;
+    r.out_swaps = out_swaps;
+    r.out_nswaps = out_nswaps;
+    r.out_status = out_status;
+    r.keys0 = at<uint32_t>(ws, L.k0);
+    r.idx0 = at<int>(ws, L.i0);
+    r.keys1 = at<uint32_t>(ws, L.k1);
+    r.idx1 = at<int>(ws, L.i1);
+    ProfScope prof(TWINKV_KERNEL_REPAIR, st);
+    return cuda_status(launch_repair(r, st));
+}
+
+}  // namespace
+}  // namespace twk
+
+using namespace twk;
+
+extern "C" {
+
+int32_t twinkv_abi_version(void) { return TWINKV_ABI_VERSION; }
+
+twinkv_params twinkv_default_params(void)
+{
+    twinkv_params p;
+    p.threshold = 0.85f;
+    p.window = 32;
+    p.n_sink = 4;
+    p.n_recent = 64;
+    return p;
+}
+
+size_t twinkv_swaps_capacity(twinkv_shape s)
+{
+    if (!shape_ok(s, false)) return 0;
+    return static_cast<size_t>(s.L) * s.H * static_cast<size_t>(s.N / 2) * 2;
+}
+
+size_t twinkv_workspace_size(twinkv_shape s, int32_t op)
+{
+    if (op < TWINKV_OP_REDUNDANCY || op > TWINKV_OP_REPAIR_SELECT) return 0;
+    if (!shape_ok(s, op != TWINKV_OP_REPAIR_SELECT)) return 0;
+    return layout(s, op).total;
+}
+
+const char* twinkv_status_string(twinkv_status st)
+{
+    switch (st) {
+    case TWINKV_OK: return "ok";
+    case TWINKV_ERR_INVALID_ARG: return "invalid argument";
+    case TWINKV_ERR_UNSUPPORTED: return "unsupported (needs an sm_103 GPU; d in {64, 128})";
+    case TWINKV_ERR_BUDGET: return "retained count differs from the budget";
+    case TWINKV_ERR_CUDA: return "CUDA error";
+    case TWINKV_ERR_TIMEOUT: return "a device-side wait timed out";
+    case TWINKV_ERR_WORKSPACE: return "workspace missing, misaligned or too small";
+    }
+    return "unknown status";
+}
+
+twinkv_status twinkv_set_wait_timeout_ns(uint64_t ns)
+{
+    if (ns == 0) return TWINKV_ERR_INVALID_ARG;
+    std::lock_guard<std::mutex> lk(g_mu);
+    g_timeout_ns = ns;
+    return TWINKV_OK;
+}
+
+twinkv_status twinkv_get_last_error(void)
+{
+    DeviceInfo* dev = nullptr;
+    const twinkv_status r = device_info(&dev);
+    if (r != TWINKV_OK) return r;
+    const cudaError_t sync = cudaDeviceSynchronize();
+    const cudaError_t last = cudaGetLastError();
+    if (sync != cudaSuccess || last != cudaSuccess) return TWINKV_ERR_CUDA;
+    int word[4];
+    if (cudaMemcpyFromSymbol(word, g_error_word, sizeof word) != cudaSuccess)
+        return TWINKV_ERR_CUDA;
+    if (word[0] != 0) {
+        const int zero[4] = {0, 0, 0, 0};
+        cudaMemcpyToSymbol(g_error_word, zero, sizeof zero);
+        return static_cast<twinkv_status>(word[0]);
+    }
+    return TWINKV_OK;
+}
+
+twinkv_status twinkv_wait_probe(uint64_t timeout_ns, int32_t* out, void* stream)
+{
+    if (!out || timeout_ns == 0) return TWINKV_ERR_INVALID_ARG;
+    DeviceInfo* dev = nullptr;
+    twinkv_status r = device_info(&dev);
+    if (r != TWINKV_OK) return r;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    if (cudaMemsetAsync(dev->probe, 0, 4 * sizeof(int), st) != cudaSuccess) return TWINKV_ERR_CUDA;
+    if (launch_wait_probe(dev->probe, timeout_ns, st) != cudaSuccess) return TWINKV_ERR_CUDA;
+    int word[4];
+    if (cudaMemcpyAsync(word, dev->probe, sizeof word, cudaMemcpyDeviceToHost, st) != cudaSuccess ||
+        cudaStreamSynchronize(st) != cudaSuccess)
+        return TWINKV_ERR_CUDA;
+    *out = word[0];
+    return TWINKV_OK;
+}
+
+twinkv_status twinkv_profile_begin(void)
+{
+    std::lock_guard<std::mutex> lk(g_mu);
+    for (auto& r : g_prof) {
+        cudaEventDestroy(r.start);
+        cudaEventDestroy(r.stop);
+    }
+    g_prof.clear();
+    g_prof_on = true;
+    return TWINKV_OK;
+}
+
+twinkv_status twinkv_profile_end(int32_t* launches, double* total_ms)
+{
+    std::vector<ProfRecord> recs;
+    {
+        std::lock_guard<std::mutex> lk(g_mu);
+        g_prof_on = false;
+        recs.swap(g_prof);
+    }
+    twinkv_status st = TWINKV_OK;
+    for (int k = 0; k < TWINKV_KERNEL_COUNT; ++k) {
+        if (launches) launches[k] = 0;
+        if (total_ms) total_ms[k] = 0.0;
+    }
+    for (auto& r : recs) {
+        float ms = 0.f;
+        if (cudaEventSynchronize(r.stop) != cudaSuccess ||
+            cudaEventElapsedTime(&ms, r.start, r.stop) != cudaSuccess)
+            st = TWINKV_ERR_CUDA;
+        if (launches) launches[r.kernel] += 1;
+        if (total_ms) total_ms[r.kernel] += ms;
+        cudaEventDestroy(r.start);
+        cudaEventDestroy(r.stop);
+    }
+    return st;
+}
+
+twinkv_status twinkv_redundancy(const void* keys, twinkv_shape s, int32_t window,
+                                float* out_score, int32_t* out_twin, void* workspace,
+                                size_t workspace_bytes, void* stream)
+{
+    if (!keys || !out_score || !out_twin || window < 0 || !shape_ok(s, true))
+        return TWINKV_ERR_INVALID_ARG;
+    Layout L;
+    twinkv_status r = check_ws(s, TWINKV_OP_REDUNDANCY, workspace, workspace_bytes, &L);
+    if (r != TWINKV_OK) return r;
+    DeviceInfo* dev = nullptr;
+    if ((r = device_info(&dev)) != TWINKV_OK) return r;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+
+    const uint16_t* k16 = nullptr;
+    if ((r = keys_bf16(keys, s, workspace, L, st, &k16)) != TWINKV_OK) return r;
+    const int U = s.L * s.H;
+    const int64_t NP = column_stride(s.N);
+    float* colrinv = at<float>(workspace, L.colrinv);
+    int* colpos = at<int>(workspace, L.colpos);
+    {
+        ProfScope p(TWINKV_KERNEL_PREP, st);
+        if (launch_norms_identity(k16, U, s.N, s.d, NP, colrinv, colpos, st) != cudaSuccess)
+            return TWINKV_ERR_CUDA;
+    }
+    AuditArgs a;
+    std::memset(&a, 0, sizeof a);
+    a.U = U;
+    a.N = s.N;
+    a.NP = static_cast<int>(NP);
+    a.RB = (s.N + kBM - 1) / kBM;
+    a.window = window < s.N ? window : s.N;
+    a.repair_mode = 0;
+    a.need_all = 0;
+    a.b_rows_per_unit = s.N;
+    a.colrinv = colrinv;
+    a.colpos = colpos;
+    a.rowrinv = colrinv;
+    a.rowrinv_stride = NP;
+    a.out_b0 = out_score;
+    a.out_t0 = out_twin;
+    a.err = dev->err;
+    a.timeout_ns = g_timeout_ns;
+    return run_audit(*dev, s, k16, k16, static_cast<int64_t>(U) * s.N, a, st);
+}
+
+twinkv_status twinkv_repair(const void* keys, twinkv_shape s, const uint8_t* retained_mask,
+                            const int32_t* budget, float threshold, const twinkv_params* params,
+                            uint8_t* out_mask, int32_t* out_swaps, int32_t* out_nswaps,
+                            float* out_score_ret, int32_t* out_twin_ret, float* out_score_all,
+                            int32_t* out_twin_all, int32_t* out_status, void* workspace,
+                            size_t workspace_bytes, void* stream)
+{
+    const twinkv_params p = params ? *params : twinkv_default_params();
+    if (!keys || !retained_mask || !out_mask || !out_nswaps || !shape_ok(s, true) ||
+        (!out_swaps && s.N >= 2))   // with N < 2 there is no room for a swap
+        return TWINKV_ERR_INVALID_ARG;
+    twinkv_status r = params_ok(p, threshold);
+    if (r != TWINKV_OK) return r;
+    Layout L;
+    if ((r = check_ws(s, TWINKV_OP_REPAIR, workspace, workspace_bytes, &L)) != TWINKV_OK) return r;
+    DeviceInfo* dev = nullptr;
+    if ((r = device_info(&dev)) != TWINKV_OK) return r;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+
+    const uint16_t* k16 = nullptr;
+    if ((r = keys_bf16(keys, s, workspace, L, st, &k16)) != TWINKV_OK) return r;
+    const int U = s.L * s.H;
+    const int64_t NP = column_stride(s.N);
+    float* colrinv = at<float>(workspace, L.colrinv);
+    int* colpos = at<int>(workspace, L.colpos);
+    uint16_t* kp = at<uint16_t>(workspace, L.kp);
+    float* rowrinv = at<float>(workspace, L.rowrinv);
+    int* cnt = at<int>(workspace, L.cnt);
+    int* kb = at<int>(workspace, L.kb);
+    {
+        ProfScope pr(TWINKV_KERNEL_PREP, st);
+        if (launch_scan(retained_mask, U, s.N, cnt, kb, st) != cudaSuccess) return TWINKV_ERR_CUDA;
+    }
+    {
+        ProfScope pr(TWINKV_KERNEL_PREP, st);
+        if (launch_gather(k16, retained_mask, cnt, kb, U, s.N, s.d, NP, kp, colrinv, colpos,
+                          rowrinv, st) != cudaSuccess)
+            return TWINKV_ERR_CUDA;
+    }
+    float* bret = out_score_ret ? out_score_ret : at<float>(workspace, L.bret);
+    AuditArgs a;
+    std::memset(&a, 0, sizeof a);
+    a.U = U;
+    a.N = s.N;
+    a.NP = static_cast<int>(NP);
+    a.RB = (s.N + kBM - 1) / kBM;
+    a.window = p.window < s.N ? p.window : s.N;
+    a.repair_mode = 1;
+    a.need_all = (out_score_all || out_twin_all) ? 1 : 0;
+    a.b_rows_per_unit = NP;
+    a.colrinv = colrinv;
+    a.colpos = colpos;
+    a.rowrinv = rowrinv;
+    a.rowrinv_stride = s.N;
+    a.cnt = cnt;
+    a.kb = kb;
+    a.out_b0 = bret;
+    a.out_t0 = out_twin_ret;
+    a.out_ball = out_score_all;
+    a.out_tall = out_twin_all;
+    a.err = dev->err;
+    a.timeout_ns = g_timeout_ns;
+    if ((r = run_audit(*dev, s, k16, kp, static_cast<int64_t>(U) * NP, a, st)) != TWINKV_OK)
+        return r;
+    return launch_select(s, bret, retained_mask, budget, threshold, p, out_mask, out_swaps,
+                         out_nswaps, out_status, workspace, L, st);
+}
+
+twinkv_status twinkv_repair_select(const float* score_ret, twinkv_shape s,
+                                   const uint8_t* retained_mask, const int32_t* budget,
+                                   float threshold, const twinkv_params* params,
+                                   uint8_t* out_mask, int32_t* out_swaps, int32_t* out_nswaps,
+                                   int32_t* out_status, void* workspace, size_t workspace_bytes,
+                                   void* stream)
+{
+    const twinkv_params p = params ? *params : twinkv_default_params();
+    if (!score_ret || !retained_mask || !out_mask || !out_nswaps || !shape_ok(s, false) ||
+        (!out_swaps && s.N >= 2))
+        return TWINKV_ERR_INVALID_ARG;
+    twinkv_status r = params_ok(p, threshold);
+    if (r != TWINKV_OK) return r;
+    Layout L;
+    if ((r = check_ws(s, TWINKV_OP_REPAIR_SELECT, workspace, workspace_bytes, &L)) != TWINKV_OK)
+        return r;
+    DeviceInfo* dev = nullptr;
+    if ((r = device_info(&dev)) != TWINKV_OK) return r;
+    return launch_select(s, score_ret, retained_mask, budget, threshold, p, out_mask, out_swaps,
+                         out_nswaps, out_status, workspace, L, static_cast<cudaStream_t>(stream));
+}
+
+}  // extern "C"

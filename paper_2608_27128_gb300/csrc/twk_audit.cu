@@ -1,0 +1,575 @@
+// twk_audit.cu -- fused redundancy audit for sm_103a (TwinKV, arXiv 2608.27128).
+//
+// For every key i of every unit it computes, without materialising the N x N matrix,
+//   Sec. 3.2 Eq. 1   sim(i,j) = k_i . k_j / (||k_i|| ||k_j||)
+//   Sec. 3.2         only j with |i - j| > w count (this also drops j = i)
+//   Sec. 3.4 Eq. 4   b_i(S0) = max over retained j, -1 if none; and its argmax
+//   (b_i(all))       the same over every j
+//
+// Design (one persistent CTA per SM, 320 threads, warp-specialised):
+//   warp 0      TMA producer: the 128-row A block of keys i (once per work item), then
+//               per 256-column tile the B tile of keys j (in 64-wide K chunks) and the
+//               tile's column metadata (1/||k_j|| and original positions).
+//   warp 1      owns TMEM (512 columns = two 128x256 fp32 accumulators) and issues
+//               tcgen05.mma (M=128, N=256, K=16, bf16 -> fp32) from one thread.
+//   warps 2..9  epilogue: warpgroup h in {0,1} takes columns [128h, 128h+128) of each
+//               tile; a thread owns one row (TMEM lane) and keeps its running maximum.
+// Keys enter the tensor cores un-normalised (bf16 products are exact in fp32);
+// 1/||k_j|| is applied per element in fp32 and 1/||k_i|| once per row after the
+// maximum (exact algebra: 1/||k_i|| > 0).
+//
+// Max and argmax in one operation: after scaling, the low 7 mantissa bits of each
+// value are replaced by (127 - c), c the column within the warpgroup's 128 columns;
+// a plain fp32 max then returns the largest value (to 2^-16 relative) and, among
+// equal truncated values, the lowest column.  Columns to ignore carry NaN (max skips
+// NaN): padding columns have 1/||k_j|| = NaN, and window columns (|i - j| <= w) are
+// set to NaN on the few tiles that intersect the window band of the row block.
+//
+// Column layout: in repair mode the columns of a unit are stored retained-first
+// (retained keys in position order, padded to a tile, then evicted keys in position
+// order), so every tile belongs to exactly one of the two maxima; the maximum over
+// all columns is the larger of the two, merged per row at the end.
+#include "twk_internal.h"
+#include "twk_ptx.cuh"
+
+namespace twk {
+namespace {
+
+constexpr int kThreads = 320;
+constexpr uint32_t kTmemCols = 512;
+constexpr uint32_t kMantMask = 0xFFFFFF80u;
+
+template <int D>
+struct AuditCfg {
+    static constexpr int KC = D / 64;                 // 128-byte K chunks per key row
+    static constexpr int A_CHUNK = kBM * 128;         // 16 KB
+    static constexpr int A_BYTES = KC * A_CHUNK;
+    static constexpr int B_STAGE = kBN * 128;         // 32 KB: one K chunk of a tile
+    static constexpr int STAGES = (D == 128) ? 4 : 5;
+    static constexpr int MSLOTS = 6;
+    static constexpr int META = kBN * 8;              // rinv[256] + pos[256]
+    static constexpr int OFF_A = 0;
+    static constexpr int OFF_B = OFF_A + 2 * A_BYTES;
+    static constexpr int OFF_META = OFF_B + STAGES * B_STAGE;
+    static constexpr int OFF_X = OFF_META + MSLOTS * META;   // 2 x 128 rows x 16 B
+    static constexpr int OFF_BAR = OFF_X + 2 * kBM * 16;
+    static constexpr int NBAR = 2 + 2 + 2 * STAGES + 2 * MSLOTS + 2 + 2 + 2 + 2 + 1;
+    static constexpr int OFF_MISC = OFF_BAR + NBAR * 8;
+    static constexpr int BYTES = OFF_MISC + 16 + 1024;       // + 1024 for alignment
+};
+
+__device__ __forceinline__ float fmax3(float a, float b, float c)
+{
+    float r;
+    asm("max.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(a), "f"(b), "f"(c));
+    return r;
+}
+
+__device__ __forceinline__ float pack(float v, uint32_t idx)
+{
+    return __uint_as_float((__float_as_uint(v) & kMantMask) | idx);
+}
+
+__device__ __forceinline__ float nan_f() { return __uint_as_float(0x7FFFFFFFu); }
+
+// 32 columns of one row: scale by 1/||k_j||, pack the column, fold into ma/mb.
+__device__ __forceinline__ void fold32(const uint32_t (&x)[32], const float* rinv, int c0,
+                                       float& ma, float& mb)
+{
+#pragma unroll
+    for (int k = 0; k < 32; k += 4) {
+        const float4 r = *reinterpret_cast<const float4*>(rinv + k);
+        const float2 p01 = __fmul2_rn(make_float2(__uint_as_float(x[k]), __uint_as_float(x[k + 1])),
+                                      make_float2(r.x, r.y));
+        const float2 p23 = __fmul2_rn(
+            make_float2(__uint_as_float(x[k + 2]), __uint_as_float(x[k + 3])),
+            make_float2(r.z, r.w));
+        const uint32_t i0 = 127u - static_cast<uint32_t>(c0 + k);
+        ma = fmax3(ma, pack(p01.x, i0), pack(p01.y, i0 - 1u));
+        mb = fmax3(mb, pack(p23.x, i0 - 2u), pack(p23.y, i0 - 3u));
+    }
+}
+
+// The same with the window test: column j is dropped when |pos_j - row| <= w,
+// i.e. when (unsigned)(pos_j - (row - w)) <= 2w.
+__device__ __forceinline__ void fold32_masked(const uint32_t (&x)[32], const float* rinv,
+                                              const int* pos, int c0, int rw, uint32_t w2,
+                                              float& ma, float& mb)
+{
+#pragma unroll
+    for (int k = 0; k < 32; k += 4) {
+        const float4 r = *reinterpret_cast<const float4*>(rinv + k);
+        const int4 p = *reinterpret_cast<const int4*>(pos + k);
+        float v0 = __uint_as_float(x[k]) * r.x;
+        float v1 = __uint_as_float(x[k + 1]) * r.y;
+        float v2 = __uint_as_float(x[k + 2]) * r.z;
+        float v3 = __uint_as_float(x[k + 3]) * r.w;
+        v0 = (static_cast<uint32_t>(p.x - rw) > w2) ? v0 : nan_f();
+        v1 = (static_cast<uint32_t>(p.y - rw) > w2) ? v1 : nan_f();
+        v2 = (static_cast<uint32_t>(p.z - rw) > w2) ? v2 : nan_f();
+        v3 = (static_cast<uint32_t>(p.w - rw) > w2) ? v3 : nan_f();
+        const uint32_t i0 = 127u - static_cast<uint32_t>(c0 + k);
+        ma = fmax3(ma, pack(v0, i0), pack(v1, i0 - 1u));
+        mb = fmax3(mb, pack(v2, i0 - 2u), pack(v3, i0 - 3u));
+    }
+}
+
+// One warpgroup's 128 columns of the accumulator for this thread's row.
+template <bool kMasked>
+__device__ __forceinline__ float half_tile(uint32_t taddr, const float* rinv, const int* pos,
+                                           int rw, uint32_t w2)
+{
+    float m0 = nan_f(), m1 = nan_f(), m2 = nan_f(), m3 = nan_f();
+#pragma unroll
+    for (int c = 0; c < 4; c += 2) {
+        uint32_t x0[32], x1[32];
+        tmem_ld_32x32b_x32(taddr + c * 32, x0);
+        tmem_ld_32x32b_x32(taddr + (c + 1) * 32, x1);
+        tmem_wait_ld();
+        if (kMasked) {
+            fold32_masked(x0, rinv + c * 32, pos + c * 32, c * 32, rw, w2, m0, m1);
+            fold32_masked(x1, rinv + (c + 1) * 32, pos + (c + 1) * 32, (c + 1) * 32, rw, w2,
+                          m2, m3);
+        } else {
+            fold32(x0, rinv + c * 32, c * 32, m0, m1);
+            fold32(x1, rinv + (c + 1) * 32, (c + 1) * 32, m2, m3);
+        }
+    }
+    return fmax3(m0, m1, fmaxf(m2, m3));
+}
+
+struct Tiles {
+    int tr;   // tiles of segment 0 (retained, or every column in mode 0)
+    int te;   // tiles of segment 1 (evicted; 0 unless b_all is wanted)
+};
+
+__device__ __forceinline__ Tiles unit_tiles(const AuditArgs& a, int u)
+{
+    if (!a.repair_mode) return {(a.N + kBN - 1) / kBN, 0};
+    const int kb = a.kb[u];
+    return {(kb + kBN - 1) / kBN, a.need_all ? (a.N - kb + kBN - 1) / kBN : 0};
+}
+
+// Lane 0 waits, the warp follows its verdict.
+__device__ __forceinline__ bool lane0_wait(uint64_t* bar, uint32_t parity, const WaitCtl& w,
+                                           int where)
+{
+    int ok = 1;
+    if ((threadIdx.x & 31) == 0) ok = mbar_wait(bar, parity, w, where) ? 1 : 0;
+    return __shfl_sync(0xFFFFFFFFu, ok, 0) != 0;
+}
+
+// Every lane waits (each needs the acquire), the warp agrees on the verdict.
+__device__ __forceinline__ bool all_wait(uint64_t* bar, uint32_t parity, const WaitCtl& w,
+                                         int where)
+{
+    const bool ok = mbar_wait(bar, parity, w, where);
+    return __all_sync(0xFFFFFFFFu, ok);
+}
+
+// Bounded wait that ignores the abort flag (used to drain in-flight copies).
+__device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity, uint64_t limit_ns)
+{
+    const uint32_t a = smem_u32(bar);
+    const uint64_t t0 = globaltimer_ns();
+    while (!mbar_try_wait(a, parity))
+        if (globaltimer_ns() - t0 > limit_ns) return;
+}
+
+// Parity of the last arming of slot s after `total` armings of a ring of `n` slots,
+// or -1 if slot s was never armed.
+__device__ __forceinline__ int last_parity(long long total, int n, int s)
+{
+    if (total <= s) return -1;
+    const long long k = s + (long long)n * ((total - 1 - s) / n);
+    return static_cast<int>((k / n) & 1);
+}
+
+template <int D>
+__global__ void __launch_bounds__(kThreads, 1)
+    audit_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                 const __grid_constant__ AuditArgs a)
+{
+    using C = AuditCfg<D>;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
+    uint8_t* sA = smem + C::OFF_A;
+    uint8_t* sB = smem + C::OFF_B;
+    uint8_t* sMeta = smem + C::OFF_META;
+    float4* sX = reinterpret_cast<float4*>(smem + C::OFF_X);
+    uint64_t* bars = reinterpret_cast<uint64_t*>(smem + C::OFF_BAR);
+    uint64_t* a_full = bars;
+    uint64_t* a_empty = a_full + 2;
+    uint64_t* b_full = a_empty + 2;
+    uint64_t* b_empty = b_full + C::STAGES;
+    uint64_t* m_full = b_empty + C::STAGES;
+    uint64_t* m_empty = m_full + C::MSLOTS;
+    uint64_t* t_full = m_empty + C::MSLOTS;
+    uint64_t* t_empty = t_full + 2;
+    uint64_t* x_full = t_empty + 2;
+    uint64_t* x_empty = x_full + 2;
+    uint64_t* drain = x_empty + 2;
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + C::OFF_MISC);
+    volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + C::OFF_MISC + 4);
+
+    const int warp = threadIdx.x >> 5;
+    const int lane = threadIdx.x & 31;
+
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(&a_full[i], 1);
+            mbar_init(&a_empty[i], 1);
+            mbar_init(&t_full[i], 1);
+            mbar_init(&t_empty[i], 8);
+            mbar_init(&x_full[i], 128);
+            mbar_init(&x_empty[i], 128);
+        }
+        for (int i = 0; i < C::STAGES; ++i) {
+            mbar_init(&b_full[i], 1);
+            mbar_init(&b_empty[i], 1);
+        }
+        for (int i = 0; i < C::MSLOTS; ++i) {
+            mbar_init(&m_full[i], 1);
+            mbar_init(&m_empty[i], 8);
+        }
+        mbar_init(drain, 1);
+        *abort_flag = 0;
+        fence_mbarrier_init();
+    }
+    if (warp == 0 && lane == 0) {
+        prefetch_tensormap(&tmA);
+        prefetch_tensormap(&tmB);
+    }
+    if (warp == 1) tmem_alloc(tmem_slot, kTmemCols);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tmem_slot;
+
+    WaitCtl wc;
+    wc.limit_ns = a.timeout_ns;
+    wc.abort_flag = abort_flag;
+    wc.err = a.err;
+    wc.where = 0;
+    const int n_items = a.U * a.RB;
+
+    if (warp == 0) {
+        // ------------------------------------------------------------ TMA producer
+        long long n_a = 0, n_b = 0, n_m = 0;
+        bool ok = true;
+        for (int item = blockIdx.x; item < n_items && ok; item += gridDim.x) {
+            const int u = item / a.RB;
+            const int rb = item - u * a.RB;
+            const Tiles ut = unit_tiles(a, u);
+            const int ab = static_cast<int>(n_a & 1);
+            ok = lane0_wait(&a_empty[ab], static_cast<uint32_t>(((n_a >> 1) & 1) ^ 1), wc, 1);
+            if (!ok) break;
+            if (lane == 0) {
+                mbar_arrive_expect_tx(&a_full[ab], C::A_BYTES);
+                const int y = u * a.N + rb * kBM;
+#pragma unroll
+                for (int kc = 0; kc < C::KC; ++kc)
+                    tma_load_2d(sA + ab * C::A_BYTES + kc * C::A_CHUNK, &tmA, &a_full[ab],
+                                kc * 64, y);
+            }
+            __syncwarp();
+            ++n_a;
+            const int nt = ut.tr + ut.te;
+            for (int t = 0; t < nt && ok; ++t) {
+                const int col0 = t * kBN;
+                const int ms = static_cast<int>(n_m % C::MSLOTS);
+                ok = lane0_wait(&m_empty[ms],
+                                static_cast<uint32_t>(((n_m / C::MSLOTS) & 1) ^ 1), wc, 2);
+                if (!ok) break;
+                if (lane == 0) {
+                    mbar_arrive_expect_tx(&m_full[ms], C::META);
+                    const int64_t off = static_cast<int64_t>(u) * a.NP + col0;
+                    bulk_load(sMeta + ms * C::META, a.colrinv + off, kBN * 4, &m_full[ms]);
+                    bulk_load(sMeta + ms * C::META + kBN * 4, a.colpos + off, kBN * 4,
+                              &m_full[ms]);
+                }
+                __syncwarp();
+                ++n_m;
+                const int yb = static_cast<int>(u * a.b_rows_per_unit + col0);
+                for (int kc = 0; kc < C::KC; ++kc) {
+                    const int s = static_cast<int>(n_b % C::STAGES);
+                    ok = lane0_wait(&b_empty[s],
+                                    static_cast<uint32_t>(((n_b / C::STAGES) & 1) ^ 1), wc, 3);
+                    if (!ok) break;
+                    if (lane == 0) {
+                        mbar_arrive_expect_tx(&b_full[s], C::B_STAGE);
+                        tma_load_2d(sB + s * C::B_STAGE, &tmB, &b_full[s], kc * 64, yb);
+                    }
+                    __syncwarp();
+                    ++n_b;
+                }
+            }
+        }
+        if (!ok && lane == 0) {
+            // Let every copy this warp started land before the block exits.
+            for (int s = 0; s < 2; ++s) {
+                const int p = last_parity(n_a, 2, s);
+                if (p >= 0) drain_wait(&a_full[s], p, a.timeout_ns);
+            }
+            for (int s = 0; s < C::STAGES; ++s) {
+                const int p = last_parity(n_b, C::STAGES, s);
+                if (p >= 0) drain_wait(&b_full[s], p, a.timeout_ns);
+            }
+            for (int s = 0; s < C::MSLOTS; ++s) {
+                const int p = last_parity(n_m, C::MSLOTS, s);
+                if (p >= 0) drain_wait(&m_full[s], p, a.timeout_ns);
+            }
+        }
+        __syncwarp();
+    } else if (warp == 1) {
+        // ------------------------------------------------------------ MMA issuer
+        constexpr uint32_t idesc = umma_idesc_bf16_f32(kBM, kBN);
+        long long n_a = 0, n_b = 0, n_t = 0;
+        bool ok = true;
+        for (int item = blockIdx.x; item < n_items && ok; item += gridDim.x) {
+            const int u = item / a.RB;
+            const Tiles ut = unit_tiles(a, u);
+            const int ab = static_cast<int>(n_a & 1);
+            ok = lane0_wait(&a_full[ab], static_cast<uint32_t>((n_a >> 1) & 1), wc, 4);
+            if (!ok) break;
+            tc_fence_after();
+            const uint32_t a_base = smem_u32(sA + ab * C::A_BYTES);
+            const int nt = ut.tr + ut.te;
+            for (int t = 0; t < nt && ok; ++t) {
+                const int acc = static_cast<int>(n_t & 1);
+                ok = lane0_wait(&t_empty[acc], static_cast<uint32_t>(((n_t >> 1) & 1) ^ 1), wc,
+                                5);
+                if (!ok) break;
+                tc_fence_after();
+                const uint32_t d_tmem = tmem + static_cast<uint32_t>(acc * kBN);
+                for (int kc = 0; kc < C::KC; ++kc) {
+                    const int s = static_cast<int>(n_b % C::STAGES);
+                    ok = lane0_wait(&b_full[s], static_cast<uint32_t>((n_b / C::STAGES) & 1), wc,
+                                    6);
+                    if (!ok) break;
+                    tc_fence_after();
+                    if (lane == 0) {
+                        const uint64_t ad = umma_desc_sw128(a_base + kc * C::A_CHUNK);
+                        const uint64_t bd = umma_desc_sw128(smem_u32(sB + s * C::B_STAGE));
+#pragma unroll
+                        for (int k = 0; k < 4; ++k)
+                            umma_bf16(d_tmem, ad + 2u * k, bd + 2u * k, idesc,
+                                      (kc | k) != 0 ? 1u : 0u);
+                        umma_commit(&b_empty[s]);
+                    }
+                    __syncwarp();
+                    ++n_b;
+                }
+                if (!ok) break;
+                if (lane == 0) umma_commit(&t_full[acc]);
+                __syncwarp();
+                ++n_t;
+            }
+            if (!ok) break;
+            if (lane == 0) umma_commit(&a_empty[ab]);
+            __syncwarp();
+            ++n_a;
+        }
+        // Every MMA this thread issued completes before TMEM is released.
+        if (lane == 0) {
+            umma_commit(drain);
+            drain_wait(drain, 0, a.timeout_ns);
+        }
+        __syncwarp();
+    } else {
+        // ------------------------------------------------------------ epilogue
+        const int ew = warp - 2;
+        const int h = ew >> 2;            // column half of the tile
+        const int q = warp & 3;           // TMEM lane quarter this warp may read
+        const int row_local = q * 32 + lane;
+        const uint32_t lane_base = static_cast<uint32_t>(q * 32) << 16;
+        const int w = a.window;
+        const uint32_t w2 = 2u * static_cast<uint32_t>(w);
+        long long n_m = 0, n_t = 0, n_x = 0;
+        bool ok = true;
+        for (int item = blockIdx.x; item < n_items && ok; item += gridDim.x) {
+            const int u = item / a.RB;
+            const int rb = item - u * a.RB;
+            const Tiles ut = unit_tiles(a, u);
+            const int nt = ut.tr + ut.te;
+            const int r0 = rb * kBM;
+            const int row = r0 + row_local;
+
+            // Column ranges that meet the window band [r0 - w, r0 + 128 + w) of this
+            // row block: only tiles meeting them need the per-element window test.
+            const int lo = max(r0 - w, 0);
+            const int hi = min(r0 + kBM + w, a.N);
+            int s0a, s0b, s1a = 0, s1b = 0;
+            if (!a.repair_mode) {
+                s0a = lo;
+                s0b = hi;
+            } else {
+                const int kb = a.kb[u];
+                const int* cnt = a.cnt + static_cast<int64_t>(u) * a.N;
+                const int clo = lo < a.N ? cnt[lo] : kb;
+                const int chi = hi < a.N ? cnt[hi] : kb;
+                const int kpad = ut.tr * kBN;
+                s0a = clo;
+                s0b = chi;
+                s1a = kpad + lo - clo;
+                s1b = kpad + hi - chi;
+            }
+
+            float bv0 = -INFINITY, bv1 = -INFINITY;   // running best of segment 0 / 1
+            int bc0 = -1, bc1 = -1;                   // and its column
+            const int rw = row - w;
+            for (int t = 0; t < nt; ++t) {
+                const int ms = static_cast<int>(n_m % C::MSLOTS);
+                const int acc = static_cast<int>(n_t & 1);
+                ok = all_wait(&m_full[ms], static_cast<uint32_t>((n_m / C::MSLOTS) & 1), wc, 7);
+                if (ok) ok = all_wait(&t_full[acc], static_cast<uint32_t>((n_t >> 1) & 1), wc, 8);
+                if (!ok) break;
+                tc_fence_after();
+                const float* rinv = reinterpret_cast<const float*>(sMeta + ms * C::META) + h * kHalf;
+                const int* pos =
+                    reinterpret_cast<const int*>(sMeta + ms * C::META + kBN * 4) + h * kHalf;
+                const int c_lo = t * kBN + h * kHalf;
+                const bool band = (c_lo < s0b && c_lo + kHalf > s0a) ||
+                                  (c_lo < s1b && c_lo + kHalf > s1a);
+                const uint32_t taddr =
+                    tmem + lane_base + static_cast<uint32_t>(acc * kBN + h * kHalf);
+                const float m = band ? half_tile<true>(taddr, rinv, pos, rw, w2)
+                                     : half_tile<false>(taddr, rinv, pos, rw, w2);
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) {
+                    mbar_arrive(&t_empty[acc]);
+                    mbar_arrive(&m_empty[ms]);
+                }
+                ++n_m;
+                ++n_t;
+                const float tv = __uint_as_float(__float_as_uint(m) & kMantMask);
+                const int tc = c_lo + 127 - static_cast<int>(__float_as_uint(m) & 127u);
+                if (t < ut.tr) {
+                    if (tv > bv0) {
+                        bv0 = tv;
+                        bc0 = tc;
+                    }
+                } else if (tv > bv1) {
+                    bv1 = tv;
+                    bc1 = tc;
+                }
+            }
+            if (!ok) break;
+
+            // Merge the two column halves of every row through shared memory.
+            const int xb = static_cast<int>(n_x & 1);
+            float4* X = sX + xb * kBM;
+            if (h == 1) {
+                ok = all_wait(&x_empty[xb], static_cast<uint32_t>(((n_x >> 1) & 1) ^ 1), wc, 9);
+                if (!ok) break;
+                X[row_local] = make_float4(bv0, __int_as_float(bc0), bv1, __int_as_float(bc1));
+                mbar_arrive(&x_full[xb]);
+            } else {
+                ok = all_wait(&x_full[xb], static_cast<uint32_t>((n_x >> 1) & 1), wc, 10);
+                if (!ok) break;
+                const float4 o = X[row_local];
+                mbar_arrive(&x_empty[xb]);
+                float v0 = bv0, v1 = bv1;
+                int c0 = bc0, c1 = bc1;
+                const int oc0 = __float_as_int(o.y), oc1 = __float_as_int(o.w);
+                if (oc0 >= 0 && (c0 < 0 || o.x > v0 || (o.x == v0 && oc0 < c0))) {
+                    v0 = o.x;
+                    c0 = oc0;
+                }
+                if (oc1 >= 0 && (c1 < 0 || o.z > v1 || (o.z == v1 && oc1 < c1))) {
+                    v1 = o.z;
+                    c1 = oc1;
+                }
+                if (row < a.N) {
+                    const int64_t o_idx = static_cast<int64_t>(u) * a.N + row;
+                    const float rr = a.rowrinv[static_cast<int64_t>(u) * a.rowrinv_stride + row];
+                    const int64_t cbase = static_cast<int64_t>(u) * a.NP;
+                    const int p0 = c0 < 0 ? -1 : (a.repair_mode ? a.colpos[cbase + c0] : c0);
+                    a.out_b0[o_idx] = p0 < 0 ? -1.0f : v0 * rr;
+                    if (a.out_t0) a.out_t0[o_idx] = p0;
+                    if (a.repair_mode && a.need_all) {
+                        const int p1 = c1 < 0 ? -1 : a.colpos[cbase + c1];
+                        const bool take1 =
+                            p1 >= 0 && (p0 < 0 || v1 > v0 || (v1 == v0 && p1 < p0));
+                        const int pb = take1 ? p1 : p0;
+                        const float vb = take1 ? v1 : v0;
+                        if (a.out_ball) a.out_ball[o_idx] = pb < 0 ? -1.0f : vb * rr;
+                        if (a.out_tall) a.out_tall[o_idx] = pb;
+                    }
+                }
+            }
+            ++n_x;
+        }
+    }
+
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (warp == 1) tmem_dealloc(tmem, kTmemCols);
+}
+
+}  // namespace
+
+size_t audit_smem_bytes(int d)
+{
+    return d == 128 ? AuditCfg<128>::BYTES : AuditCfg<64>::BYTES;
+}
+
+cudaError_t launch_audit(int d, const CUtensorMap& tmA, const CUtensorMap& tmB,
+                         const AuditArgs& a, int grid, cudaStream_t st)
+{
+    if (d == 128) {
+        const int bytes = AuditCfg<128>::BYTES;
+        cudaError_t e = cudaFuncSetAttribute(audit_kernel<128>,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+        if (e != cudaSuccess) return e;
+        audit_kernel<128><<<grid, kThreads, bytes, st>>>(tmA, tmB, a);
+    } else {
+        const int bytes = AuditCfg<64>::BYTES;
+        cudaError_t e = cudaFuncSetAttribute(audit_kernel<64>,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+        if (e != cudaSuccess) return e;
+        audit_kernel<64><<<grid, kThreads, bytes, st>>>(tmA, tmB, a);
+    }
+    return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------- wait probe
+
+namespace {
+__global__ void wait_probe_kernel(int* err, unsigned long long timeout_ns)
+{
+    __shared__ uint64_t bar;
+    __shared__ uint32_t slot;
+    __shared__ int abort_flag;
+    if (threadIdx.x == 0) {
+        mbar_init(&bar, 1);
+        abort_flag = 0;
+        fence_mbarrier_init();
+    }
+    if (threadIdx.x < 32) tmem_alloc(&slot, 32);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    WaitCtl wc;
+    wc.limit_ns = timeout_ns;
+    wc.abort_flag = &abort_flag;
+    wc.err = err;
+    wc.where = 0;
+    // Nothing ever arrives on `bar`: its phase 0 never completes.
+    (void)mbar_wait(&bar, 0, wc, 99);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (threadIdx.x < 32) tmem_dealloc(slot, 32);
+}
+}  // namespace
+
+cudaError_t launch_wait_probe(int* err, unsigned long long timeout_ns, cudaStream_t st)
+{
+    wait_probe_kernel<<<1, 64, 0, st>>>(err, timeout_ns);
+    return cudaGetLastError();
+}
+
+}  // namespace twk

@@ -1,0 +1,261 @@
+// twk_repair.cu -- budget-exact repair swap of TwinKV (arXiv 2608.27128, Sec. 3.4).
+//
+// One block of 1024 threads per unit (layer, KV head):
+//   1. validate S0: every mask byte in {0,1}, popcount == budget (when given);
+//   2. classify  orphan = i not in S0 and b_i < tau,
+//                donor  = j in S0, outside [0, n_sink) and [N - n_recent, N), b_j >= tau;
+//   3. compact both lists in position order (warp ballots + a block scan), each entry a
+//      (severity key, position) pair: orphans keyed by b ascending, donors by b
+//      descending, through an order-preserving float -> u32 map (-0 folded into +0);
+//   4. stable LSD radix sort of each list (8-bit digits, warp match + per-warp digit
+//      counts), so equal severities keep position order (lower position first);
+//   5. m = min(|O|, |D|): S1 = S0 with the first m donors cleared and the first m
+//      orphans set; swaps[k] = (donor k, orphan k).
+// Sort buffers are caller workspace ([U][N] keys and positions, twice).
+#include "twk_internal.h"
+
+namespace twk {
+namespace {
+
+constexpr int kT = 1024;
+constexpr int kW = kT / 32;
+
+__device__ __forceinline__ uint32_t ordered(float b)
+{
+    uint32_t u = __float_as_uint(b == 0.0f ? 0.0f : b);
+    return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+
+struct Shared {
+    int warp_cnt[kW][256];   // per-warp digit counts, then their prefix over warps
+    int base[256];           // running output offset of each digit
+    int chunk_tot[256];
+    int wsum[2][kW];         // block-scan scratch for the two lists
+    int red[4];
+    int flag;
+};
+
+// Block-wide exclusive scan of two 0/1 flags; returns the prefixes and the chunk totals.
+__device__ __forceinline__ void scan2(Shared& s, int fo, int fd, int& po, int& pd, int& to,
+                                      int& td)
+{
+    const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+    const uint32_t bo = __ballot_sync(0xFFFFFFFFu, fo);
+    const uint32_t bd = __ballot_sync(0xFFFFFFFFu, fd);
+    const uint32_t lt = (1u << lane) - 1u;
+    if (lane == 0) {
+        s.wsum[0][wid] = __popc(bo);
+        s.wsum[1][wid] = __popc(bd);
+    }
+    __syncthreads();
+    if (wid == 0) {
+        int a = s.wsum[0][lane], b = s.wsum[1][lane];
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int ya = __shfl_up_sync(0xFFFFFFFFu, a, o);
+            const int yb = __shfl_up_sync(0xFFFFFFFFu, b, o);
+            if (lane >= o) {
+                a += ya;
+                b += yb;
+            }
+        }
+        s.wsum[0][lane] = a;   // inclusive
+        s.wsum[1][lane] = b;
+    }
+    __syncthreads();
+    po = (wid ? s.wsum[0][wid - 1] : 0) + __popc(bo & lt);
+    pd = (wid ? s.wsum[1][wid - 1] : 0) + __popc(bd & lt);
+    to = s.wsum[0][kW - 1];
+    td = s.wsum[1][kW - 1];
+    __syncthreads();
+}
+
+// One stable counting pass on digit (key >> shift) & 255 of n items; returns false
+// (and moves nothing) when every item has the same digit.
+__device__ bool radix_pass(Shared& s, const uint32_t* kin, const int* iin, uint32_t* kout,
+                           int* iout, int n, int shift)
+{
+    const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+    for (int i = threadIdx.x; i < kW * 256; i += kT) (&s.warp_cnt[0][0])[i] = 0;
+    if (threadIdx.x < 256) s.base[threadIdx.x] = 0;
+    __syncthreads();
+    for (int c0 = 0; c0 < n; c0 += kT) {
+        const int i = c0 + threadIdx.x;
+        const int dg = i < n ? static_cast<int>((kin[i] >> shift) & 255) : 256;
+        const uint32_t peers = __match_any_sync(0xFFFFFFFFu, dg);
+        if (dg < 256 && lane == __ffs(peers) - 1) atomicAdd(&s.base[dg], __popc(peers));
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        int run = 0, single = 0;
+        for (int d = 0; d < 256; ++d) {
+            const int c = s.base[d];
+            if (c == n) single = 1;
+            s.base[d] = run;
+            run += c;
+        }
+        s.flag = single;
+    }
+    __syncthreads();
+    if (s.flag) return false;
+    for (int c0 = 0; c0 < n; c0 += kT) {
+        const int i = c0 + threadIdx.x;
+        const bool valid = i < n;
+        const uint32_t key = valid ? kin[i] : 0u;
+        const int dg = valid ? static_cast<int>((key >> shift) & 255) : 256;
+        const uint32_t peers = __match_any_sync(0xFFFFFFFFu, dg);
+        const int rank = __popc(peers & ((1u << lane) - 1u));
+        if (valid && rank == 0) s.warp_cnt[wid][dg] = __popc(peers);
+        __syncthreads();
+        if (threadIdx.x < 256) {
+            int run = 0;
+            for (int w = 0; w < kW; ++w) {
+                const int t = s.warp_cnt[w][threadIdx.x];
+                s.warp_cnt[w][threadIdx.x] = run;
+                run += t;
+            }
+            s.chunk_tot[threadIdx.x] = run;
+        }
+        __syncthreads();
+        if (valid) {
+            const int dst = s.base[dg] + s.warp_cnt[wid][dg] + rank;
+            kout[dst] = key;
+            iout[dst] = iin[i];
+        }
+        __syncthreads();
+        if (threadIdx.x < 256) {
+            s.base[threadIdx.x] += s.chunk_tot[threadIdx.x];
+            for (int w = 0; w < kW; ++w) s.warp_cnt[w][threadIdx.x] = 0;
+        }
+        __syncthreads();
+    }
+    return true;
+}
+
+// Sorts n (key, position) items held at offset `off` of buffer 0; returns the buffer
+// (0 or 1) that holds the sorted result.
+__device__ int radix_sort(Shared& s, uint32_t* k0, int* i0, uint32_t* k1, int* i1, int n)
+{
+    int cur = 0;
+    for (int shift = 0; shift < 32; shift += 8) {
+        const bool moved = cur == 0 ? radix_pass(s, k0, i0, k1, i1, n, shift)
+                                    : radix_pass(s, k1, i1, k0, i0, n, shift);
+        if (moved) cur ^= 1;
+        __syncthreads();
+    }
+    return cur;
+}
+
+__global__ void __launch_bounds__(kT, 1) repair_kernel(const RepairArgs a)
+{
+    __shared__ Shared s;
+    const int u = blockIdx.x;
+    const int N = a.N;
+    const int64_t off = static_cast<int64_t>(u) * N;
+    const uint8_t* S0 = a.mask + off;
+    const float* b = a.b + off;
+    uint8_t* S1 = a.out_mask + off;
+    int* swaps = a.out_swaps + static_cast<int64_t>(u) * 2 * (N / 2);
+
+    // 1. validation
+    int bad = 0, cnt = 0, no = 0, nd = 0;
+    const float tau = a.tau;
+    for (int i = threadIdx.x; i < N; i += kT) {
+        const uint8_t v = S0[i];
+        bad |= v > 1;
+        cnt += v != 0;
+        const bool prot = i < a.n_sink || i >= N - a.n_recent;
+        no += (v == 0 && b[i] < tau);
+        nd += (v != 0 && !prot && b[i] >= tau);
+    }
+    if (threadIdx.x < 4) s.red[threadIdx.x] = 0;
+    __syncthreads();
+    bad = __reduce_or_sync(0xFFFFFFFFu, bad);
+    cnt = __reduce_add_sync(0xFFFFFFFFu, cnt);
+    no = __reduce_add_sync(0xFFFFFFFFu, no);
+    nd = __reduce_add_sync(0xFFFFFFFFu, nd);
+    if ((threadIdx.x & 31) == 0) {
+        atomicOr(&s.red[0], bad);
+        atomicAdd(&s.red[1], cnt);
+        atomicAdd(&s.red[2], no);
+        atomicAdd(&s.red[3], nd);
+    }
+    __syncthreads();
+    int status = 0;
+    if (s.red[0]) status = 1;                                   // TWINKV_ERR_INVALID_ARG
+    else if (a.budget && a.budget[u] != s.red[1]) status = 3;   // TWINKV_ERR_BUDGET
+    const int n_o = s.red[2], n_d = s.red[3];
+    const int m = status ? 0 : min(n_o, n_d);
+
+    // S1 starts as S0 (also the answer for a failed unit or m = 0).
+    for (int i = threadIdx.x; i < N; i += kT) S1[i] = S0[i];
+    if (status != 0 || m == 0) {
+        if (threadIdx.x == 0) {
+            a.out_nswaps[u] = status ? -1 : 0;
+            if (a.out_status) a.out_status[u] = status;
+        }
+        return;
+    }
+
+    // 2-3. classify and compact: orphans at [0, n_o), donors at [n_o, n_o + n_d)
+    uint32_t* k0 = a.keys0 + off;
+    int* i0 = a.idx0 + off;
+    uint32_t* k1 = a.keys1 + off;
+    int* i1 = a.idx1 + off;
+    int base_o = 0, base_d = n_o;
+    for (int c0 = 0; c0 < N; c0 += kT) {
+        const int i = c0 + threadIdx.x;
+        int fo = 0, fd = 0;
+        float bi = 0.f;
+        if (i < N) {
+            const uint8_t v = S0[i];
+            bi = b[i];
+            const bool prot = i < a.n_sink || i >= N - a.n_recent;
+            fo = (v == 0 && bi < tau);
+            fd = (v != 0 && !prot && bi >= tau);
+        }
+        int po, pd, to, td;
+        scan2(s, fo, fd, po, pd, to, td);
+        if (fo) {
+            k0[base_o + po] = ordered(bi);
+            i0[base_o + po] = i;
+        }
+        if (fd) {
+            k0[base_d + pd] = ~ordered(bi);
+            i0[base_d + pd] = i;
+        }
+        base_o += to;
+        base_d += td;
+    }
+    __syncthreads();
+
+    // 4. severity order
+    const int co = radix_sort(s, k0, i0, k1, i1, n_o);
+    const int cd = radix_sort(s, k0 + n_o, i0 + n_o, k1 + n_o, i1 + n_o, n_d);
+    const int* orph = co ? i1 : i0;
+    const int* don = (cd ? i1 : i0) + n_o;
+    __syncthreads();
+
+    // 5. swap
+    for (int k = threadIdx.x; k < m; k += kT) {
+        const int out_ = don[k], in_ = orph[k];
+        S1[out_] = 0;
+        S1[in_] = 1;
+        swaps[2 * k] = out_;
+        swaps[2 * k + 1] = in_;
+    }
+    if (threadIdx.x == 0) {
+        a.out_nswaps[u] = m;
+        if (a.out_status) a.out_status[u] = 0;
+    }
+}
+
+}  // namespace
+
+cudaError_t launch_repair(const RepairArgs& a, cudaStream_t st)
+{
+    repair_kernel<<<a.U, kT, 0, st>>>(a);
+    return cudaGetLastError();
+}
+
+}  // namespace twk
