@@ -9,7 +9,12 @@
  * CUDA library.
  *
  * What it computes, by paper passage:
- *   Sec. 3.2, Eq. 1      sim(i,j) = khat_i . khat_j with khat_i = k_i / ||k_i||_2
+ *   Sec. 3.2, Eq. 1      sim(i,j) = khat_i . khat_j with khat_i = k_i / ||k_i||_2,
+ *                        evaluated as (k_i . k_j) / sqrt((k_i . k_i)(k_j . k_j)): the dot
+ *                        products of bf16 keys are exact in double (16-bit products,
+ *                        d <= 128 terms), so one rounding each remains for the product,
+ *                        the square root and the quotient; the value is symmetric in
+ *                        (i, j) and exactly 1 for positively scaled duplicates
  *   Sec. 3.2, twin rule  j is a twin candidate of i only if |i-j| > w (and j != i)
  *   Sec. 3.4, Eq. 4      b_i(S0) = max over j in S0, |i-j| > w, j != i of sim(i,j);
  *                        -1 when no such j exists
@@ -68,50 +73,30 @@ void twk_oracle_round_bf16(const float* in, uint16_t* out, long n)
 
 /* ---- Eq. 1 ------------------------------------------------------------------------ */
 
-/* khat = k / ||k||_2 for every key of one (layer, head); zero keys stay zero. */
-static void normalise_keys(const uint16_t* keys, int N, int d, double* khat)
-{
-    for (int i = 0; i < N; ++i) {
-        double sq = 0.0;
-        for (int t = 0; t < d; ++t) {
-            double v = bf16_to_double(keys[(long)i * d + t]);
-            sq += v * v;
-        }
-        double norm = sqrt(sq);
-        for (int t = 0; t < d; ++t) {
-            double v = bf16_to_double(keys[(long)i * d + t]);
-            khat[(long)i * d + t] = (norm > 0.0) ? v / norm : 0.0;
-        }
-    }
-}
-
-static double dot(const double* a, const double* b, int d)
+/* k_i . k_j in double, terms in increasing t. */
+static double dot_bf16(const uint16_t* a, const uint16_t* b, int d)
 {
     double s = 0.0;
     for (int t = 0; t < d; ++t)
-        s += a[t] * b[t];
+        s += bf16_to_double(a[t]) * bf16_to_double(b[t]);
     return s;
+}
+
+/* sim(i,j) of Eq. 1 from the dot product and the two squared norms; a zero key has
+ * similarity 0 with every key. */
+static double cosine(double dot_ij, double sq_i, double sq_j)
+{
+    if (sq_i == 0.0 || sq_j == 0.0)
+        return 0.0;
+    return dot_ij / sqrt(sq_i * sq_j);
 }
 
 /* sim(i, j) of Eq. 1 for keys i and j of one (layer, head) stored as bf16 rows of
  * length d.  Used by the comparator to score a candidate twin. */
 double twk_oracle_sim(const uint16_t* key_i, const uint16_t* key_j, int d)
 {
-    double ni = 0.0, nj = 0.0;
-    for (int t = 0; t < d; ++t) {
-        double a = bf16_to_double(key_i[t]), b = bf16_to_double(key_j[t]);
-        ni += a * a;
-        nj += b * b;
-    }
-    ni = sqrt(ni);
-    nj = sqrt(nj);
-    double s = 0.0;
-    for (int t = 0; t < d; ++t) {
-        double a = (ni > 0.0) ? bf16_to_double(key_i[t]) / ni : 0.0;
-        double b = (nj > 0.0) ? bf16_to_double(key_j[t]) / nj : 0.0;
-        s += a * b;
-    }
-    return s;
+    return cosine(dot_bf16(key_i, key_j, d), dot_bf16(key_i, key_i, d),
+                  dot_bf16(key_j, key_j, d));
 }
 
 /* ---- Eq. 4 and the best twin over all keys ------------------------------------- */
@@ -140,11 +125,12 @@ void twk_oracle_audit(const uint16_t* keys, int U, int N, int d, const uint8_t* 
 {
     if (rows == NULL)
         nrows = N;
-    double* khat = (double*)malloc(sizeof(double) * (size_t)N * (size_t)d);
+    double* sq = (double*)malloc(sizeof(double) * (size_t)(N > 0 ? N : 1));
     for (int u = 0; u < U; ++u) {
         const uint16_t* K = keys + (long)u * N * d;
         const uint8_t* S0 = mask ? mask + (long)u * N : NULL;
-        normalise_keys(K, N, d, khat);
+        for (int i = 0; i < N; ++i)
+            sq[i] = dot_bf16(&K[(long)i * d], &K[(long)i * d], d);
 #pragma omp parallel for schedule(dynamic, 8)
         for (int r = 0; r < nrows; ++r) {
             int i = rows ? rows[r] : r;
@@ -156,7 +142,7 @@ void twk_oracle_audit(const uint16_t* keys, int U, int N, int d, const uint8_t* 
                 int dist = (i > j) ? i - j : j - i;
                 if (j == i || dist <= window)
                     continue;
-                double s = dot(&khat[(long)i * d], &khat[(long)j * d], d);
+                double s = cosine(dot_bf16(&K[(long)i * d], &K[(long)j * d], d), sq[i], sq[j]);
                 if (arg < 0 || s > best) {
                     if (arg >= 0)
                         second = best;
@@ -189,7 +175,7 @@ void twk_oracle_audit(const uint16_t* keys, int U, int N, int d, const uint8_t* 
             }
         }
     }
-    free(khat);
+    free(sq);
 }
 
 /* ---- Sec. 3.4: orphans, donors, severity ranking and the swap ------------------ */

@@ -337,3 +337,21 @@ def test_f32_entry_equals_f64_entry_on_float_values(oracle_mod):
     r64 = oracle_mod.repair(b.astype(np.float64), S0, 0.85)
     for k in r32:
         np.testing.assert_array_equal(r32[k], r64[k])
+
+
+def test_similarity_is_symmetric_and_exact_for_duplicates(oracle_mod):
+    """Eq. 1 is symmetric in (i, j): mutual twins carry bitwise-equal b; duplicates
+    (also positively scaled by a power of two) score exactly 1."""
+    keys = synth.random_keys(13, 1, 400, 128)
+    keys[0, 300] = keys[0, 10]
+    x = synth.bf16_bits_to_f32(keys[0, 20]) * 4.0
+    keys[0, 350] = synth.f32_to_bf16_bits(x)
+    a = oracle_mod.audit(keys, window=32)
+    t, b = a["t_all"][0], a["b_all"][0]
+    mutual = [i for i in range(400) if t[t[i]] == i]
+    assert len(mutual) > 10
+    for i in mutual:
+        assert b[i] == b[t[i]]
+    assert b[10] == 1.0 and t[10] == 300 and b[20] == 1.0 and t[20] == 350
+    for i, j in [(3, 77), (200, 5), (10, 300)]:
+        assert oracle_mod.sim(keys, 0, i, j) == oracle_mod.sim(keys, 0, j, i)
