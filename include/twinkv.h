@@ -34,7 +34,7 @@
  * aligned).  Tensors are dense, row-major, innermost dimension last:
  *   keys        [L][H][N][d]   bf16 (raw 16-bit patterns) or float32
  *   masks       [L][H][N]      uint8, 0 = evicted, 1 = retained
- *   scores      [L][H][N]      float32
+ *   scores      [L][H][N]      float64 (b values, see "Precision" below)
  *   twins       [L][H][N]      int32 position in 0..N-1, or -1
  *   per-unit    [L*H]          int32
  *   swaps       [L*H][N/2][2]  int32 pairs (evicted donor, admitted orphan); unit u's
@@ -53,6 +53,13 @@
  * gets out_nswaps[u] = -1 and out_mask equal to its input mask.  A device-side wait
  * that gives up (TWINKV_ERR_TIMEOUT) and asynchronous CUDA errors are reported by
  * twinkv_get_last_error().  No call throws, traps or aborts the process.
+ *
+ * Precision.  The twin of each key is the argmax of fp32 tensor-core similarities
+ * (bf16 products, fp32 accumulation); candidates within ~2^-16 relative of each other
+ * are not told apart.  The reported b of that twin is then recomputed as
+ * (k_i . k_j) / sqrt((k_i . k_i)(k_j . k_j)) with double-float dot products (relative
+ * error ~1e-13) and fp64 rounding, so it is symmetric in (i, j) and exactly 1 for a
+ * duplicate; orphan/donor decisions and the severity ranking use these fp64 values.
  *
  * Limits: d in {64, 128}; 1 <= N <= 1048576; L*H*N*d < 2^31 elements per tensor
  * coordinate; L*H*(N rounded up to 256, plus 256) < 2^31 rows.
@@ -107,7 +114,8 @@ typedef enum {
     TWINKV_KERNEL_PREP = 0,      /* bf16 rounding, norms, retained-first column gather */
     TWINKV_KERNEL_AUDIT = 1,     /* fused similarity + masked max/argmax (Eq. 1, Eq. 4) */
     TWINKV_KERNEL_REPAIR = 2,    /* classify, rank, select and swap (Sec. 3.4) */
-    TWINKV_KERNEL_COUNT = 3
+    TWINKV_KERNEL_REFINE = 3,    /* exact value of each chosen twin's similarity (Eq. 1) */
+    TWINKV_KERNEL_COUNT = 4
 } twinkv_kernel;
 
 /* Paper defaults: tau = 0.85, w = 32, 4 sink and 64 recent positions (Sec. 3.2). */
@@ -123,19 +131,19 @@ size_t twinkv_workspace_size(twinkv_shape s, int32_t op);
  * Best twin of every key over all other keys (Sec. 3.2, Eq. 1 and the twin window;
  * the maximum b_i(all) behind the redundancy count of Eq. 2: r_i > 0 iff
  * b_i(all) > tau).
- *   keys       [L][H][N][d] device, dtype per s.dtype
+ *   keys       [L][H][N][d] device, dtype per s.dtype, 16-byte aligned
  *   window     w >= 0
- *   out_score  [L][H][N] float32: b_i(all), or -1 when no position lies beyond w
+ *   out_score  [L][H][N] float64: b_i(all), or -1 when no position lies beyond w
  *   out_twin   [L][H][N] int32: its position (lowest on ties), or -1
  */
 twinkv_status twinkv_redundancy(const void* keys, twinkv_shape s, int32_t window,
-                                float* out_score, int32_t* out_twin, void* workspace,
+                                double* out_score, int32_t* out_twin, void* workspace,
                                 size_t workspace_bytes, void* stream);
 
 /*
  * Audit of a retained set and the budget-exact repair swap (Sec. 3.4, Eq. 4 and the
  * orphan/donor rule), all units in one pass.
- *   keys           [L][H][N][d] device
+ *   keys           [L][H][N][d] device, 16-byte aligned
  *   retained_mask  [L][H][N] uint8, S0
  *   budget         [L*H] int32 expected |S0| per unit, or NULL (no check)
  *   threshold      tau (finite); overrides params->threshold
@@ -145,9 +153,9 @@ twinkv_status twinkv_redundancy(const void* keys, twinkv_shape s, int32_t window
  *   out_swaps      [L*H][N/2][2] int32: (evicted donor, admitted orphan), most severe
  *                  first; entries past out_nswaps[u] are left untouched
  *   out_nswaps     [L*H] int32: m, or -1 for a unit with a data error
- *   out_score_ret  [L][H][N] float32 b_i(S0), or NULL
+ *   out_score_ret  [L][H][N] float64 b_i(S0), or NULL
  *   out_twin_ret   [L][H][N] int32 argmax of b_i(S0), or NULL
- *   out_score_all  [L][H][N] float32 b_i(all), or NULL; when both this and
+ *   out_score_all  [L][H][N] float64 b_i(all), or NULL; when both this and
  *                  out_twin_all are NULL the evicted columns are skipped entirely
  *                  (O(N K d) instead of O(N^2 d), Sec. 3.5)
  *   out_twin_all   [L][H][N] int32, or NULL
@@ -156,17 +164,18 @@ twinkv_status twinkv_redundancy(const void* keys, twinkv_shape s, int32_t window
 twinkv_status twinkv_repair(const void* keys, twinkv_shape s, const uint8_t* retained_mask,
                             const int32_t* budget, float threshold,
                             const twinkv_params* params, uint8_t* out_mask,
-                            int32_t* out_swaps, int32_t* out_nswaps, float* out_score_ret,
-                            int32_t* out_twin_ret, float* out_score_all,
+                            int32_t* out_swaps, int32_t* out_nswaps, double* out_score_ret,
+                            int32_t* out_twin_ret, double* out_score_all,
                             int32_t* out_twin_all, int32_t* out_status, void* workspace,
                             size_t workspace_bytes, void* stream);
 
 /*
  * The classification, ranking and swap of twinkv_repair alone, on caller-supplied
  * b_i(S0) values (Sec. 3.4).  Same arguments and outputs as twinkv_repair; s.d and
- * s.dtype are ignored.  score_ret [L][H][N] float32 device.
+ * s.dtype are ignored.  score_ret [L][H][N] float64 device.  Orphans compare
+ * b < (double)threshold, donors b >= (double)threshold.
  */
-twinkv_status twinkv_repair_select(const float* score_ret, twinkv_shape s,
+twinkv_status twinkv_repair_select(const double* score_ret, twinkv_shape s,
                                    const uint8_t* retained_mask, const int32_t* budget,
                                    float threshold, const twinkv_params* params,
                                    uint8_t* out_mask, int32_t* out_swaps,

@@ -134,8 +134,8 @@ bool shape_ok(const twinkv_shape& s, bool need_d)
 size_t up256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
 
 struct Layout {
-    size_t keys16 = 0, colrinv = 0, colpos = 0, kp = 0, rowrinv = 0, cnt = 0, kb = 0,
-           bret = 0, k0 = 0, i0 = 0, k1 = 0, i1 = 0;
+    size_t keys16 = 0, colrinv = 0, colpos = 0, norm2 = 0, kp = 0, cnt = 0, kb = 0, twin0 = 0,
+           twin1 = 0, bret = 0, k0 = 0, i0 = 0, k1 = 0, i1 = 0;
     size_t total = 0;
 };
 
@@ -155,18 +155,20 @@ Layout layout(const twinkv_shape& s, int op)
         if (s.dtype == TWINKV_F32) L.keys16 = take(U * N * s.d * 2);
         L.colrinv = take(U * NP * 4);
         L.colpos = take(U * NP * 4);
+        L.norm2 = take(U * N * 8);
         if (op == TWINKV_OP_REPAIR) {
             L.kp = take(U * NP * s.d * 2);
-            L.rowrinv = take(U * N * 4);
             L.cnt = take(U * N * 4);
             L.kb = take(U * 4);
-            L.bret = take(U * N * 4);
+            L.twin0 = take(U * N * 4);
+            L.twin1 = take(U * N * 4);
+            L.bret = take(U * N * 8);
         }
     }
     if (op == TWINKV_OP_REPAIR || op == TWINKV_OP_REPAIR_SELECT) {
-        L.k0 = take(U * N * 4);
+        L.k0 = take(U * N * 8);
         L.i0 = take(U * N * 4);
-        L.k1 = take(U * N * 4);
+        L.k1 = take(U * N * 8);
         L.i1 = take(U * N * 4);
     }
     L.total = off;
@@ -226,7 +228,7 @@ twinkv_status params_ok(const twinkv_params& p, float threshold)
     return TWINKV_OK;
 }
 
-twinkv_status launch_select(const twinkv_shape& s, const float* b, const uint8_t* mask,
+twinkv_status launch_select(const twinkv_shape& s, const double* b, const uint8_t* mask,
                             const int32_t* budget, float threshold, const twinkv_params& p,
                             uint8_t* out_mask, int32_t* out_swaps, int32_t* out_nswaps,
                             int32_t* out_status, void* ws, const Layout& L, cudaStream_t st)
@@ -237,20 +239,37 @@ twinkv_status launch_select(const twinkv_shape& s, const float* b, const uint8_t
     r.b = b;
     r.mask = mask;
     r.budget = budget;
-    r.tau = threshold;
+    r.tau = static_cast<double>(threshold);
     r.n_sink = p.n_sink;
     r.n_recent = p.n_recent;
     r.out_mask = out_mask;
     r.out_swaps = out_swaps;
     r.out_nswaps = out_nswaps;
     r.out_status = out_status;
-    r.keys0 = at<uint32_t>(ws, L.k0);
+    r.keys0 = at<uint64_t>(ws, L.k0);
     r.idx0 = at<int>(ws, L.i0);
-    r.keys1 = at<uint32_t>(ws, L.k1);
+    r.keys1 = at<uint64_t>(ws, L.k1);
     r.idx1 = at<int>(ws, L.i1);
     ProfScope prof(TWINKV_KERNEL_REPAIR, st);
     return cuda_status(launch_repair(r, st));
 }
+
+twinkv_status run_norm2(const uint16_t* k16, const twinkv_shape& s, double* norm2,
+                        cudaStream_t st)
+{
+    ProfScope p(TWINKV_KERNEL_PREP, st);
+    return cuda_status(
+        launch_norm2(k16, static_cast<int64_t>(s.L) * s.H * s.N, s.d, norm2, st));
+}
+
+twinkv_status run_refine(const uint16_t* k16, const twinkv_shape& s, const double* norm2,
+                         const int* t0, int* t1, double* b0, double* b1, cudaStream_t st)
+{
+    ProfScope p(TWINKV_KERNEL_REFINE, st);
+    return cuda_status(launch_refine(k16, s.L * s.H, s.N, s.d, norm2, t0, t1, b0, b1, st));
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; }
 
 }  // namespace
 }  // namespace twk
@@ -381,10 +400,10 @@ twinkv_status twinkv_profile_end(int32_t* launches, double* total_ms)
 }
 
 twinkv_status twinkv_redundancy(const void* keys, twinkv_shape s, int32_t window,
-                                float* out_score, int32_t* out_twin, void* workspace,
+                                double* out_score, int32_t* out_twin, void* workspace,
                                 size_t workspace_bytes, void* stream)
 {
-    if (!keys || !out_score || !out_twin || window < 0 || !shape_ok(s, true))
+    if (!keys || !aligned16(keys) || !out_score || !out_twin || window < 0 || !shape_ok(s, true))
         return TWINKV_ERR_INVALID_ARG;
     Layout L;
     twinkv_status r = check_ws(s, TWINKV_OP_REDUNDANCY, workspace, workspace_bytes, &L);
@@ -399,11 +418,13 @@ twinkv_status twinkv_redundancy(const void* keys, twinkv_shape s, int32_t window
     const int64_t NP = column_stride(s.N);
     float* colrinv = at<float>(workspace, L.colrinv);
     int* colpos = at<int>(workspace, L.colpos);
+    double* norm2 = at<double>(workspace, L.norm2);
     {
         ProfScope p(TWINKV_KERNEL_PREP, st);
         if (launch_norms_identity(k16, U, s.N, s.d, NP, colrinv, colpos, st) != cudaSuccess)
             return TWINKV_ERR_CUDA;
     }
+    if ((r = run_norm2(k16, s, norm2, st)) != TWINKV_OK) return r;
     AuditArgs a;
     std::memset(&a, 0, sizeof a);
     a.U = U;
@@ -416,25 +437,24 @@ twinkv_status twinkv_redundancy(const void* keys, twinkv_shape s, int32_t window
     a.b_rows_per_unit = s.N;
     a.colrinv = colrinv;
     a.colpos = colpos;
-    a.rowrinv = colrinv;
-    a.rowrinv_stride = NP;
-    a.out_b0 = out_score;
     a.out_t0 = out_twin;
     a.err = dev->err;
     a.timeout_ns = g_timeout_ns;
-    return run_audit(*dev, s, k16, k16, static_cast<int64_t>(U) * s.N, a, st);
+    if ((r = run_audit(*dev, s, k16, k16, static_cast<int64_t>(U) * s.N, a, st)) != TWINKV_OK)
+        return r;
+    return run_refine(k16, s, norm2, out_twin, nullptr, out_score, nullptr, st);
 }
 
 twinkv_status twinkv_repair(const void* keys, twinkv_shape s, const uint8_t* retained_mask,
                             const int32_t* budget, float threshold, const twinkv_params* params,
                             uint8_t* out_mask, int32_t* out_swaps, int32_t* out_nswaps,
-                            float* out_score_ret, int32_t* out_twin_ret, float* out_score_all,
+                            double* out_score_ret, int32_t* out_twin_ret, double* out_score_all,
                             int32_t* out_twin_all, int32_t* out_status, void* workspace,
                             size_t workspace_bytes, void* stream)
 {
     const twinkv_params p = params ? *params : twinkv_default_params();
-    if (!keys || !retained_mask || !out_mask || !out_nswaps || !shape_ok(s, true) ||
-        (!out_swaps && s.N >= 2))   // with N < 2 there is no room for a swap
+    if (!keys || !aligned16(keys) || !retained_mask || !out_mask || !out_nswaps ||
+        !shape_ok(s, true) || (!out_swaps && s.N >= 2))   // with N < 2 no swap fits
         return TWINKV_ERR_INVALID_ARG;
     twinkv_status r = params_ok(p, threshold);
     if (r != TWINKV_OK) return r;
@@ -450,8 +470,8 @@ twinkv_status twinkv_repair(const void* keys, twinkv_shape s, const uint8_t* ret
     const int64_t NP = column_stride(s.N);
     float* colrinv = at<float>(workspace, L.colrinv);
     int* colpos = at<int>(workspace, L.colpos);
+    double* norm2 = at<double>(workspace, L.norm2);
     uint16_t* kp = at<uint16_t>(workspace, L.kp);
-    float* rowrinv = at<float>(workspace, L.rowrinv);
     int* cnt = at<int>(workspace, L.cnt);
     int* kb = at<int>(workspace, L.kb);
     {
@@ -461,10 +481,14 @@ twinkv_status twinkv_repair(const void* keys, twinkv_shape s, const uint8_t* ret
     {
         ProfScope pr(TWINKV_KERNEL_PREP, st);
         if (launch_gather(k16, retained_mask, cnt, kb, U, s.N, s.d, NP, kp, colrinv, colpos,
-                          rowrinv, st) != cudaSuccess)
+                          st) != cudaSuccess)
             return TWINKV_ERR_CUDA;
     }
-    float* bret = out_score_ret ? out_score_ret : at<float>(workspace, L.bret);
+    if ((r = run_norm2(k16, s, norm2, st)) != TWINKV_OK) return r;
+    const bool need_all = out_score_all || out_twin_all;
+    int* t0 = out_twin_ret ? out_twin_ret : at<int>(workspace, L.twin0);
+    int* t1 = need_all ? (out_twin_all ? out_twin_all : at<int>(workspace, L.twin1)) : nullptr;
+    double* bret = out_score_ret ? out_score_ret : at<double>(workspace, L.bret);
     AuditArgs a;
     std::memset(&a, 0, sizeof a);
     a.U = U;
@@ -473,27 +497,25 @@ twinkv_status twinkv_repair(const void* keys, twinkv_shape s, const uint8_t* ret
     a.RB = (s.N + kBM - 1) / kBM;
     a.window = p.window < s.N ? p.window : s.N;
     a.repair_mode = 1;
-    a.need_all = (out_score_all || out_twin_all) ? 1 : 0;
+    a.need_all = need_all ? 1 : 0;
     a.b_rows_per_unit = NP;
     a.colrinv = colrinv;
     a.colpos = colpos;
-    a.rowrinv = rowrinv;
-    a.rowrinv_stride = s.N;
     a.cnt = cnt;
     a.kb = kb;
-    a.out_b0 = bret;
-    a.out_t0 = out_twin_ret;
-    a.out_ball = out_score_all;
-    a.out_tall = out_twin_all;
+    a.out_t0 = t0;
+    a.out_t1 = t1;
     a.err = dev->err;
     a.timeout_ns = g_timeout_ns;
     if ((r = run_audit(*dev, s, k16, kp, static_cast<int64_t>(U) * NP, a, st)) != TWINKV_OK)
+        return r;
+    if ((r = run_refine(k16, s, norm2, t0, t1, bret, out_score_all, st)) != TWINKV_OK)
         return r;
     return launch_select(s, bret, retained_mask, budget, threshold, p, out_mask, out_swaps,
                          out_nswaps, out_status, workspace, L, st);
 }
 
-twinkv_status twinkv_repair_select(const float* score_ret, twinkv_shape s,
+twinkv_status twinkv_repair_select(const double* score_ret, twinkv_shape s,
                                    const uint8_t* retained_mask, const int32_t* budget,
                                    float threshold, const twinkv_params* params,
                                    uint8_t* out_mask, int32_t* out_swaps, int32_t* out_nswaps,

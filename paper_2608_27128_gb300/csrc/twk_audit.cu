@@ -15,20 +15,23 @@
 //   warps 2..9  epilogue: warpgroup h in {0,1} takes columns [128h, 128h+128) of each
 //               tile; a thread owns one row (TMEM lane) and keeps its running maximum.
 // Keys enter the tensor cores un-normalised (bf16 products are exact in fp32);
-// 1/||k_j|| is applied per element in fp32 and 1/||k_i|| once per row after the
-// maximum (exact algebra: 1/||k_i|| > 0).
+// 1/||k_j|| is applied per element in fp32.  1/||k_i|| > 0 does not change the argmax
+// over j, so it is never applied: this kernel outputs the twin positions, and the
+// exact similarity of each chosen twin is computed afterwards (twk_refine.cu).
 //
 // Max and argmax in one operation: after scaling, the low 7 mantissa bits of each
 // value are replaced by (127 - c), c the column within the warpgroup's 128 columns;
-// a plain fp32 max then returns the largest value (to 2^-16 relative) and, among
-// equal truncated values, the lowest column.  Columns to ignore carry NaN (max skips
+// a plain fp32 max then returns the largest value (to 2^-16 relative, which decides
+// the argmax only among near-equal candidates) and, among equal truncated values,
+// the lowest column.  Columns to ignore carry NaN (max skips
 // NaN): padding columns have 1/||k_j|| = NaN, and window columns (|i - j| <= w) are
 // set to NaN on the few tiles that intersect the window band of the row block.
 //
 // Column layout: in repair mode the columns of a unit are stored retained-first
 // (retained keys in position order, padded to a tile, then evicted keys in position
-// order), so every tile belongs to exactly one of the two maxima; the maximum over
-// all columns is the larger of the two, merged per row at the end.
+// order), so every tile belongs to exactly one of the two maxima.  The kernel writes
+// both winners; the maximum over all columns is the larger of the two, taken on the
+// exact similarities computed afterwards.
 #include "twk_internal.h"
 #include "twk_ptx.cuh"
 
@@ -72,10 +75,39 @@ __device__ __forceinline__ float pack(float v, uint32_t idx)
 
 __device__ __forceinline__ float nan_f() { return __uint_as_float(0x7FFFFFFFu); }
 
-// 32 columns of one row: scale by 1/||k_j||, pack the column, fold into ma/mb.
-__device__ __forceinline__ void fold32(const uint32_t (&x)[32], const float* rinv, int c0,
-                                       float& ma, float& mb)
+// Orders every later use of x after the preceding tcgen05.wait::ld: the registers
+// written by tcgen05.ld are only valid after the wait, which the compiler cannot see.
+__device__ __forceinline__ void reg_fence(uint32_t (&x)[32])
 {
+    asm volatile(""
+                 : "+r"(x[0]), "+r"(x[1]), "+r"(x[2]), "+r"(x[3]), "+r"(x[4]), "+r"(x[5]),
+                   "+r"(x[6]), "+r"(x[7]), "+r"(x[8]), "+r"(x[9]), "+r"(x[10]), "+r"(x[11]),
+                   "+r"(x[12]), "+r"(x[13]), "+r"(x[14]), "+r"(x[15]), "+r"(x[16]),
+                   "+r"(x[17]), "+r"(x[18]), "+r"(x[19]), "+r"(x[20]), "+r"(x[21]),
+                   "+r"(x[22]), "+r"(x[23]), "+r"(x[24]), "+r"(x[25]), "+r"(x[26]),
+                   "+r"(x[27]), "+r"(x[28]), "+r"(x[29]), "+r"(x[30]), "+r"(x[31]));
+}
+
+// Maximum of 32 packed values as a tree of 3-input maxima (depth 4).
+__device__ __forceinline__ float tree32(const float (&p)[32])
+{
+    float q[11];
+#pragma unroll
+    for (int j = 0; j < 10; ++j) q[j] = fmax3(p[3 * j], p[3 * j + 1], p[3 * j + 2]);
+    q[10] = fmaxf(p[30], p[31]);
+    const float r0 = fmax3(q[0], q[1], q[2]);
+    const float r1 = fmax3(q[3], q[4], q[5]);
+    const float r2 = fmax3(q[6], q[7], q[8]);
+    const float r3 = fmaxf(q[9], q[10]);
+    return fmax3(r0, r1, fmaxf(r2, r3));
+}
+
+// 32 columns [c0, c0 + 32) of one row: scale by 1/||k_j||, pack the column, reduce.
+template <bool kMasked>
+__device__ __forceinline__ float fold32(const uint32_t (&x)[32], const float* rinv,
+                                        const int* pos, int c0, int rw, uint32_t w2)
+{
+    float p[32];
 #pragma unroll
     for (int k = 0; k < 32; k += 4) {
         const float4 r = *reinterpret_cast<const float4*>(rinv + k);
@@ -84,57 +116,45 @@ __device__ __forceinline__ void fold32(const uint32_t (&x)[32], const float* rin
         const float2 p23 = __fmul2_rn(
             make_float2(__uint_as_float(x[k + 2]), __uint_as_float(x[k + 3])),
             make_float2(r.z, r.w));
+        float v0 = p01.x, v1 = p01.y, v2 = p23.x, v3 = p23.y;
+        if (kMasked) {
+            // column j is dropped when |pos_j - row| <= w, i.e. (unsigned)(pos_j - (row - w)) <= 2w
+            const int4 q = *reinterpret_cast<const int4*>(pos + k);
+            v0 = (static_cast<uint32_t>(q.x - rw) > w2) ? v0 : nan_f();
+            v1 = (static_cast<uint32_t>(q.y - rw) > w2) ? v1 : nan_f();
+            v2 = (static_cast<uint32_t>(q.z - rw) > w2) ? v2 : nan_f();
+            v3 = (static_cast<uint32_t>(q.w - rw) > w2) ? v3 : nan_f();
+        }
         const uint32_t i0 = 127u - static_cast<uint32_t>(c0 + k);
-        ma = fmax3(ma, pack(p01.x, i0), pack(p01.y, i0 - 1u));
-        mb = fmax3(mb, pack(p23.x, i0 - 2u), pack(p23.y, i0 - 3u));
+        p[k] = pack(v0, i0);
+        p[k + 1] = pack(v1, i0 - 1u);
+        p[k + 2] = pack(v2, i0 - 2u);
+        p[k + 3] = pack(v3, i0 - 3u);
     }
+    return tree32(p);
 }
 
-// The same with the window test: column j is dropped when |pos_j - row| <= w,
-// i.e. when (unsigned)(pos_j - (row - w)) <= 2w.
-__device__ __forceinline__ void fold32_masked(const uint32_t (&x)[32], const float* rinv,
-                                              const int* pos, int c0, int rw, uint32_t w2,
-                                              float& ma, float& mb)
-{
-#pragma unroll
-    for (int k = 0; k < 32; k += 4) {
-        const float4 r = *reinterpret_cast<const float4*>(rinv + k);
-        const int4 p = *reinterpret_cast<const int4*>(pos + k);
-        float v0 = __uint_as_float(x[k]) * r.x;
-        float v1 = __uint_as_float(x[k + 1]) * r.y;
-        float v2 = __uint_as_float(x[k + 2]) * r.z;
-        float v3 = __uint_as_float(x[k + 3]) * r.w;
-        v0 = (static_cast<uint32_t>(p.x - rw) > w2) ? v0 : nan_f();
-        v1 = (static_cast<uint32_t>(p.y - rw) > w2) ? v1 : nan_f();
-        v2 = (static_cast<uint32_t>(p.z - rw) > w2) ? v2 : nan_f();
-        v3 = (static_cast<uint32_t>(p.w - rw) > w2) ? v3 : nan_f();
-        const uint32_t i0 = 127u - static_cast<uint32_t>(c0 + k);
-        ma = fmax3(ma, pack(v0, i0), pack(v1, i0 - 1u));
-        mb = fmax3(mb, pack(v2, i0 - 2u), pack(v3, i0 - 3u));
-    }
-}
-
-// One warpgroup's 128 columns of the accumulator for this thread's row.
+// One warpgroup's 128 columns of the accumulator for this thread's row: the second
+// pair of TMEM loads is in flight while the first pair is reduced.
 template <bool kMasked>
 __device__ __forceinline__ float half_tile(uint32_t taddr, const float* rinv, const int* pos,
                                            int rw, uint32_t w2)
 {
-    float m0 = nan_f(), m1 = nan_f(), m2 = nan_f(), m3 = nan_f();
-#pragma unroll
-    for (int c = 0; c < 4; c += 2) {
-        uint32_t x0[32], x1[32];
-        tmem_ld_32x32b_x32(taddr + c * 32, x0);
-        tmem_ld_32x32b_x32(taddr + (c + 1) * 32, x1);
-        tmem_wait_ld();
-        if (kMasked) {
-            fold32_masked(x0, rinv + c * 32, pos + c * 32, c * 32, rw, w2, m0, m1);
-            fold32_masked(x1, rinv + (c + 1) * 32, pos + (c + 1) * 32, (c + 1) * 32, rw, w2,
-                          m2, m3);
-        } else {
-            fold32(x0, rinv + c * 32, c * 32, m0, m1);
-            fold32(x1, rinv + (c + 1) * 32, (c + 1) * 32, m2, m3);
-        }
-    }
+    uint32_t x0[32], x1[32], x2[32], x3[32];
+    tmem_ld_32x32b_x32(taddr, x0);
+    tmem_ld_32x32b_x32(taddr + 32, x1);
+    tmem_wait_ld();
+    reg_fence(x0);
+    reg_fence(x1);
+    tmem_ld_32x32b_x32(taddr + 64, x2);
+    tmem_ld_32x32b_x32(taddr + 96, x3);
+    const float m0 = fold32<kMasked>(x0, rinv, pos, 0, rw, w2);
+    const float m1 = fold32<kMasked>(x1, rinv + 32, pos + 32, 32, rw, w2);
+    tmem_wait_ld();
+    reg_fence(x2);
+    reg_fence(x3);
+    const float m2 = fold32<kMasked>(x2, rinv + 64, pos + 64, 64, rw, w2);
+    const float m3 = fold32<kMasked>(x3, rinv + 96, pos + 96, 96, rw, w2);
     return fmax3(m0, m1, fmaxf(m2, m3));
 }
 
@@ -470,7 +490,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (!ok) break;
                 const float4 o = X[row_local];
                 mbar_arrive(&x_empty[xb]);
-                float v0 = bv0, v1 = bv1;
+                float v0 = bv0, v1 = bv1;   // truncated values decide only within a half
                 int c0 = bc0, c1 = bc1;
                 const int oc0 = __float_as_int(o.y), oc1 = __float_as_int(o.w);
                 if (oc0 >= 0 && (c0 < 0 || o.x > v0 || (o.x == v0 && oc0 < c0))) {
@@ -483,20 +503,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
                 if (row < a.N) {
                     const int64_t o_idx = static_cast<int64_t>(u) * a.N + row;
-                    const float rr = a.rowrinv[static_cast<int64_t>(u) * a.rowrinv_stride + row];
                     const int64_t cbase = static_cast<int64_t>(u) * a.NP;
                     const int p0 = c0 < 0 ? -1 : (a.repair_mode ? a.colpos[cbase + c0] : c0);
-                    a.out_b0[o_idx] = p0 < 0 ? -1.0f : v0 * rr;
-                    if (a.out_t0) a.out_t0[o_idx] = p0;
-                    if (a.repair_mode && a.need_all) {
-                        const int p1 = c1 < 0 ? -1 : a.colpos[cbase + c1];
-                        const bool take1 =
-                            p1 >= 0 && (p0 < 0 || v1 > v0 || (v1 == v0 && p1 < p0));
-                        const int pb = take1 ? p1 : p0;
-                        const float vb = take1 ? v1 : v0;
-                        if (a.out_ball) a.out_ball[o_idx] = pb < 0 ? -1.0f : vb * rr;
-                        if (a.out_tall) a.out_tall[o_idx] = pb;
-                    }
+                    a.out_t0[o_idx] = p0;
+                    if (a.repair_mode && a.need_all)
+                        a.out_t1[o_idx] = c1 < 0 ? -1 : a.colpos[cbase + c1];
                 }
             }
             ++n_x;

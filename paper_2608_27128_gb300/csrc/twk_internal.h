@@ -24,32 +24,29 @@ struct AuditArgs {
     int64_t b_rows_per_unit;    // row stride of a unit in the B tensor map
     const float* colrinv;       // [U][NP]  1/||k|| per column, NaN on padding columns
     const int* colpos;          // [U][NP]  original position of each column
-    const float* rowrinv;       // [U][rowrinv_stride]  1/||k_i|| per row
-    int64_t rowrinv_stride;
-    const int* cnt;             // [U][N]  retained positions before p (repair mode)
-    const int* kb;              // [U]     |S0| (repair mode)
-    float* out_b0;              // [U][N]  segment-0 best (b_ret, or b_all in mode 0)
-    int* out_t0;                // nullable
-    float* out_ball;            // [U][N]  repair mode, nullable
-    int* out_tall;              // nullable
+    const int* cnt;             // [U][N]   retained positions before p (repair mode)
+    const int* kb;              // [U]      |S0| (repair mode)
+    int* out_t0;                // [U][N]   argmax of segment 0 (retained, or all in mode 0)
+    int* out_t1;                // [U][N]   argmax of segment 1, the evicted columns
+                                //          (repair mode with need_all), -1 if none
     int* err;
     unsigned long long timeout_ns;
 };
 
 struct RepairArgs {
     int U, N;
-    const float* b;             // [U][N] b_i(S0)
+    const double* b;            // [U][N] b_i(S0)
     const uint8_t* mask;        // [U][N]
     const int* budget;          // [U] or null
-    float tau;
+    double tau;                 // threshold rounded to float, widened
     int n_sink, n_recent;
     uint8_t* out_mask;          // [U][N]
     int* out_swaps;             // [U][N/2][2]
     int* out_nswaps;            // [U]
     int* out_status;            // [U] or null
-    uint32_t* keys0;            // [U][N] sort buffers (ping-pong)
+    uint64_t* keys0;            // [U][N] sort buffers (ping-pong)
     int* idx0;
-    uint32_t* keys1;
+    uint64_t* keys1;
     int* idx1;
 };
 
@@ -60,7 +57,15 @@ cudaError_t launch_norms_identity(const uint16_t* keys, int U, int N, int d, int
 cudaError_t launch_scan(const uint8_t* mask, int U, int N, int* cnt, int* kb, cudaStream_t st);
 cudaError_t launch_gather(const uint16_t* keys, const uint8_t* mask, const int* cnt,
                           const int* kb, int U, int N, int d, int64_t NP, uint16_t* kp,
-                          float* colrinv, int* colpos, float* rowrinv, cudaStream_t st);
+                          float* colrinv, int* colpos, cudaStream_t st);
+
+// exact similarity of the chosen twins
+cudaError_t launch_norm2(const uint16_t* keys, int64_t n, int d, double* norm2, cudaStream_t st);
+// b0 = sim(i, twin0); with twin1 given (the evicted-segment winner), twin1 is
+// overwritten with the overall winner and b1 (nullable) receives its similarity.
+cudaError_t launch_refine(const uint16_t* keys, int U, int N, int d, const double* norm2,
+                          const int* twin0, int* twin1, double* b0, double* b1,
+                          cudaStream_t st);
 
 // audit kernel (tensor maps built by the caller)
 size_t audit_smem_bytes(int d);

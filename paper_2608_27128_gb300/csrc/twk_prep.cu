@@ -117,8 +117,7 @@ template <int D>
 __global__ void gather_kernel(const uint16_t* __restrict__ keys, const uint8_t* __restrict__ mask,
                               const int* __restrict__ cnt, const int* __restrict__ kb, int U,
                               int N, int64_t NP, uint16_t* __restrict__ kp,
-                              float* __restrict__ colrinv, int* __restrict__ colpos,
-                              float* __restrict__ rowrinv)
+                              float* __restrict__ colrinv, int* __restrict__ colpos)
 {
     const int64_t total = static_cast<int64_t>(U) * NP;   // N positions + NP-N padding per unit
     const int64_t wstride = static_cast<int64_t>(gridDim.x) * (blockDim.x >> 5);
@@ -141,7 +140,6 @@ __global__ void gather_kernel(const uint16_t* __restrict__ keys, const uint8_t* 
             if (lane == 0) {
                 colrinv[u * NP + col] = r;
                 colpos[u * NP + col] = p;
-                rowrinv[u * N + p] = r;
             }
         } else {
             // padding columns: [k, kpad) and [kpad + N - k, NP)
@@ -196,15 +194,15 @@ cudaError_t launch_scan(const uint8_t* mask, int U, int N, int* cnt, int* kb, cu
 
 cudaError_t launch_gather(const uint16_t* keys, const uint8_t* mask, const int* cnt,
                           const int* kb, int U, int N, int d, int64_t NP, uint16_t* kp,
-                          float* colrinv, int* colpos, float* rowrinv, cudaStream_t st)
+                          float* colrinv, int* colpos, cudaStream_t st)
 {
     const int grid = grid_for(static_cast<int64_t>(U) * NP, 8);
     if (d == 128)
         gather_kernel<128><<<grid, 256, 0, st>>>(keys, mask, cnt, kb, U, N, NP, kp, colrinv,
-                                                 colpos, rowrinv);
+                                                 colpos);
     else
         gather_kernel<64><<<grid, 256, 0, st>>>(keys, mask, cnt, kb, U, N, NP, kp, colrinv,
-                                                colpos, rowrinv);
+                                                colpos);
     return cudaGetLastError();
 }
 

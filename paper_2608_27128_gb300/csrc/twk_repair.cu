@@ -6,9 +6,10 @@
 //                donor  = j in S0, outside [0, n_sink) and [N - n_recent, N), b_j >= tau;
 //   3. compact both lists in position order (warp ballots + a block scan), each entry a
 //      (severity key, position) pair: orphans keyed by b ascending, donors by b
-//      descending, through an order-preserving float -> u32 map (-0 folded into +0);
+//      descending, through an order-preserving fp64 -> u64 map (-0 folded into +0);
 //   4. stable LSD radix sort of each list (8-bit digits, warp match + per-warp digit
-//      counts), so equal severities keep position order (lower position first);
+//      counts; a digit position shared by every key is skipped), so equal severities
+//      keep position order (lower position first);
 //   5. m = min(|O|, |D|): S1 = S0 with the first m donors cleared and the first m
 //      orphans set; swaps[k] = (donor k, orphan k).
 // Sort buffers are caller workspace ([U][N] keys and positions, twice).
@@ -20,10 +21,10 @@ namespace {
 constexpr int kT = 1024;
 constexpr int kW = kT / 32;
 
-__device__ __forceinline__ uint32_t ordered(float b)
+__device__ __forceinline__ uint64_t ordered(double b)
 {
-    uint32_t u = __float_as_uint(b == 0.0f ? 0.0f : b);
-    return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+    const uint64_t u = static_cast<uint64_t>(__double_as_longlong(b == 0.0 ? 0.0 : b));
+    return (u >> 63) ? ~u : (u | 0x8000000000000000ull);
 }
 
 struct Shared {
@@ -72,7 +73,7 @@ __device__ __forceinline__ void scan2(Shared& s, int fo, int fd, int& po, int& p
 
 // One stable counting pass on digit (key >> shift) & 255 of n items; returns false
 // (and moves nothing) when every item has the same digit.
-__device__ bool radix_pass(Shared& s, const uint32_t* kin, const int* iin, uint32_t* kout,
+__device__ bool radix_pass(Shared& s, const uint64_t* kin, const int* iin, uint64_t* kout,
                            int* iout, int n, int shift)
 {
     const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
@@ -101,7 +102,7 @@ __device__ bool radix_pass(Shared& s, const uint32_t* kin, const int* iin, uint3
     for (int c0 = 0; c0 < n; c0 += kT) {
         const int i = c0 + threadIdx.x;
         const bool valid = i < n;
-        const uint32_t key = valid ? kin[i] : 0u;
+        const uint64_t key = valid ? kin[i] : 0ull;
         const int dg = valid ? static_cast<int>((key >> shift) & 255) : 256;
         const uint32_t peers = __match_any_sync(0xFFFFFFFFu, dg);
         const int rank = __popc(peers & ((1u << lane) - 1u));
@@ -134,10 +135,10 @@ __device__ bool radix_pass(Shared& s, const uint32_t* kin, const int* iin, uint3
 
 // Sorts n (key, position) items held at offset `off` of buffer 0; returns the buffer
 // (0 or 1) that holds the sorted result.
-__device__ int radix_sort(Shared& s, uint32_t* k0, int* i0, uint32_t* k1, int* i1, int n)
+__device__ int radix_sort(Shared& s, uint64_t* k0, int* i0, uint64_t* k1, int* i1, int n)
 {
     int cur = 0;
-    for (int shift = 0; shift < 32; shift += 8) {
+    for (int shift = 0; shift < 64; shift += 8) {
         const bool moved = cur == 0 ? radix_pass(s, k0, i0, k1, i1, n, shift)
                                     : radix_pass(s, k1, i1, k0, i0, n, shift);
         if (moved) cur ^= 1;
@@ -153,13 +154,13 @@ __global__ void __launch_bounds__(kT, 1) repair_kernel(const RepairArgs a)
     const int N = a.N;
     const int64_t off = static_cast<int64_t>(u) * N;
     const uint8_t* S0 = a.mask + off;
-    const float* b = a.b + off;
+    const double* b = a.b + off;
     uint8_t* S1 = a.out_mask + off;
     int* swaps = a.out_swaps + static_cast<int64_t>(u) * 2 * (N / 2);
 
     // 1. validation
     int bad = 0, cnt = 0, no = 0, nd = 0;
-    const float tau = a.tau;
+    const double tau = a.tau;
     for (int i = threadIdx.x; i < N; i += kT) {
         const uint8_t v = S0[i];
         bad |= v > 1;
@@ -198,15 +199,15 @@ __global__ void __launch_bounds__(kT, 1) repair_kernel(const RepairArgs a)
     }
 
     // 2-3. classify and compact: orphans at [0, n_o), donors at [n_o, n_o + n_d)
-    uint32_t* k0 = a.keys0 + off;
+    uint64_t* k0 = a.keys0 + off;
     int* i0 = a.idx0 + off;
-    uint32_t* k1 = a.keys1 + off;
+    uint64_t* k1 = a.keys1 + off;
     int* i1 = a.idx1 + off;
     int base_o = 0, base_d = n_o;
     for (int c0 = 0; c0 < N; c0 += kT) {
         const int i = c0 + threadIdx.x;
         int fo = 0, fd = 0;
-        float bi = 0.f;
+        double bi = 0.0;
         if (i < N) {
             const uint8_t v = S0[i];
             bi = b[i];

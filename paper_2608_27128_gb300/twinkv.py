@@ -21,8 +21,8 @@ from . import build as _build
 OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_BUDGET, ERR_CUDA, ERR_TIMEOUT, ERR_WORKSPACE = range(7)
 BF16, F32 = 0, 1
 OP_REDUNDANCY, OP_REPAIR, OP_REPAIR_SELECT = 0, 1, 2
-KERNEL_PREP, KERNEL_AUDIT, KERNEL_REPAIR = 0, 1, 2
-KERNEL_NAMES = ("prep", "audit", "repair")
+KERNEL_PREP, KERNEL_AUDIT, KERNEL_REPAIR, KERNEL_REFINE = 0, 1, 2, 3
+KERNEL_NAMES = ("prep", "audit", "repair", "refine")
 
 EXPORTED = (
     "twinkv_abi_version", "twinkv_default_params", "twinkv_swaps_capacity",
@@ -184,13 +184,13 @@ def twinkv_redundancy(keys, window: int = 32, out_score=None, out_twin=None, ws=
                       stream=None):
     """Best twin of every key over all other keys outside the +-window band.
 
-    keys: [L,H,N,d] bf16/float32 CUDA tensor.  Returns (score f32 [L,H,N],
+    keys: [L,H,N,d] bf16/float32 CUDA tensor.  Returns (score float64 [L,H,N],
     twin int32 [L,H,N]); score = -1 and twin = -1 where no position lies beyond w.
     """
     s = shape_of(keys)
     dev = keys.device
     _need(keys, "keys", keys.dtype, keys.shape, dev)
-    out_score = _out(out_score, "out_score", torch.float32, keys.shape[:3], dev)
+    out_score = _out(out_score, "out_score", torch.float64, keys.shape[:3], dev)
     out_twin = _out(out_twin, "out_twin", torch.int32, keys.shape[:3], dev)
     ws = _ws(ws, s, OP_REDUNDANCY, dev)
     st = load().twinkv_redundancy(_ptr(keys), s, int(window), _ptr(out_score), _ptr(out_twin),
@@ -239,10 +239,10 @@ def twinkv_repair(keys, retained_mask, budget=None, threshold=None, params=None,
         "status": _out(out.get("status"), "status", torch.int32, (L * H,), dev),
     }
     if want_ret:
-        o["score_ret"] = _out(out.get("score_ret"), "score_ret", torch.float32, (L, H, N), dev)
+        o["score_ret"] = _out(out.get("score_ret"), "score_ret", torch.float64, (L, H, N), dev)
         o["twin_ret"] = _out(out.get("twin_ret"), "twin_ret", torch.int32, (L, H, N), dev)
     if want_all:
-        o["score_all"] = _out(out.get("score_all"), "score_all", torch.float32, (L, H, N), dev)
+        o["score_all"] = _out(out.get("score_all"), "score_all", torch.float64, (L, H, N), dev)
         o["twin_all"] = _out(out.get("twin_all"), "twin_all", torch.int32, (L, H, N), dev)
     ws = _ws(ws, s, OP_REPAIR, dev)
     st = load().twinkv_repair(
@@ -257,12 +257,12 @@ def twinkv_repair(keys, retained_mask, budget=None, threshold=None, params=None,
 def twinkv_repair_select(score_ret, retained_mask, budget=None, threshold=None, params=None,
                          *, n_sink=None, n_recent=None, out=None, ws=None,
                          stream=None) -> dict:
-    """The classification, ranking and swap alone, on given b_i(S0) values [L,H,N]."""
+    """The classification, ranking and swap alone, on given float64 b_i(S0) [L,H,N]."""
     if score_ret.dim() != 3:
         raise ValueError("score_ret must be [L, H, N]")
     L, H, N = (int(x) for x in score_ret.shape)
     dev = score_ret.device
-    _need(score_ret, "score_ret", torch.float32, (L, H, N), dev)
+    _need(score_ret, "score_ret", torch.float64, (L, H, N), dev)
     _need(retained_mask, "retained_mask", torch.uint8, (L, H, N), dev)
     if budget is not None:
         _need(budget, "budget", torch.int32, (L * H,), dev)
@@ -304,7 +304,8 @@ def twinkv_profile_begin():
 
 
 def twinkv_profile_end() -> dict:
-    n = (ctypes.c_int32 * 3)()
-    ms = (ctypes.c_double * 3)()
+    k = len(KERNEL_NAMES)
+    n = (ctypes.c_int32 * k)()
+    ms = (ctypes.c_double * k)()
     _check(load().twinkv_profile_end(n, ms), "twinkv_profile_end")
-    return {KERNEL_NAMES[k]: (int(n[k]), float(ms[k])) for k in range(3)}
+    return {KERNEL_NAMES[i]: (int(n[i]), float(ms[i])) for i in range(k)}

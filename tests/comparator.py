@@ -19,6 +19,8 @@ class Report:
     n_fail: int = 0
     n_excused: int = 0
     notes: list = field(default_factory=list)
+    # largest |b_gpu - b_oracle| over rows whose twin agrees (the refined value)
+    max_dev_same_twin: float = 0.0
 
     def fail(self, msg):
         self.n_fail += 1
@@ -28,6 +30,7 @@ class Report:
     def add(self, other):
         self.n_fail += other.n_fail
         self.n_excused += other.n_excused
+        self.max_dev_same_twin = max(self.max_dev_same_twin, other.max_dev_same_twin)
         self.notes += other.notes[: max(0, 20 - len(self.notes))]
         return self
 
@@ -52,6 +55,7 @@ def compare_best(b_gpu, t_gpu, b_orc, t_orc, b_orc2, sim, window, rows=None, S0=
         if abs(bg - bo) > TOL:
             rep.fail(f"{what} row {i}: score {bg} vs {bo}")
         if tg == to:
+            rep.max_dev_same_twin = max(rep.max_dev_same_twin, abs(bg - bo))
             continue
         ok = (0 <= tg and abs(tg - i) > window and (S0 is None or S0[tg])
               and bo - b2 <= BAND and sim(i, tg) >= bo - BAND)

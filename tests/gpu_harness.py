@@ -74,8 +74,10 @@ def repair_vs_oracle(keys, S0, L, H, window, tau, n_sink=4, n_recent=64, want_al
 
 
 def split_check(h, S0, tau, n_sink, n_recent, budget=None):
+    """The oracle's repair fed the GPU's own fp64 b_ret must reproduce S1, the swap
+    lists and their lengths bit for bit."""
     U, N = S0.shape
-    rf = oracle.repair_f32(h["score_ret"].reshape(U, N), S0, tau, n_sink=n_sink,
+    rf = oracle.repair(h["score_ret"].reshape(U, N), S0, tau, n_sink=n_sink,
                            n_recent=n_recent,
                            budget=S0.sum(1) if budget is None else budget)
     np.testing.assert_array_equal(h["nswaps"], rf["nswaps"])

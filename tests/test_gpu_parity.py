@@ -88,6 +88,7 @@ def test_redundancy_matches_oracle(L, H, N, d, w):
     rep, s, t = redundancy_vs_oracle(keys, L, H, w)
     assert rep.n_fail == 0, rep.notes
     assert rep.n_excused <= max(1, N // 100)
+    assert rep.max_dev_same_twin < 1e-9
 
 
 REPAIR_CASES = [
@@ -112,6 +113,7 @@ def test_repair_matches_oracle(L, H, N, d, w, K, tau, ns, nr):
     S0 = synth.random_masks(41 + N, L * H, N, K)
     rep, h, a, r = repair_vs_oracle(keys, S0, L, H, w, tau, ns, nr)
     assert rep.n_fail == 0, rep.notes
+    assert rep.max_dev_same_twin < 1e-9
 
 
 def test_repair_without_b_all_skips_nothing_it_reports():
@@ -161,6 +163,7 @@ def test_workload_recipes(name, over, ratio):
     S0 = synth.masks(w, ratio)
     rep, h, a, r = repair_vs_oracle(keys, S0, w.L, w.H, synth.WINDOW, w.tau)
     assert rep.n_fail == 0, rep.notes
+    assert rep.max_dev_same_twin < 1e-9
     if name == "tiny":
         assert rep.n_excused == 0, rep.notes
     # planted twins are found exactly, with no tie excuse
@@ -184,9 +187,10 @@ def test_repair_select_is_bit_exact(seed):
     rng = np.random.default_rng(seed)
     L, H, N = 2, 3, int(rng.integers(50, 5000))
     U = L * H
-    grid = np.array([-1.0, -0.0, 0.0, 0.25, 0.5, 0.75, 0.85, 0.9, 1.0], np.float32)
+    grid = np.array([-1.0, -0.0, 0.0, 0.25, 0.5, 0.75, 0.85, 0.9, 1.0,
+                     float(np.float32(0.5)) + 1e-12])
     b = np.where(rng.random((U, N)) < 0.5, rng.choice(grid, size=(U, N)),
-                 rng.uniform(-1, 1, size=(U, N))).astype(np.float32)
+                 rng.uniform(-1, 1, size=(U, N)))
     S0 = synth.random_masks(seed, U, N, N // 2)
     tau = 0.5
     budget = S0.sum(1).astype(np.int32)

@@ -1,0 +1,145 @@
+"""The four large workloads at full size, in the launch configuration bench.py times
+(one twinkv_repair call over every layer and head, with b_i(all)).
+
+Checked per workload:
+  * every unit: the bit-exact split check (oracle repair on the GPU's own b_i(S0)), the
+    budget and swap invariants of Sec. 3.4, and the planted ground truth (twins of
+    planted pairs farther apart than w; evicted needles admitted as orphans);
+  * a few whole units: full comparison with the fp64 oracle (scores, twins, S1, swaps);
+  * the long workload: a random 4096-row sample per head against the oracle.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from comparator import Report, compare_best, compare_repair
+from gpu_harness import device, keys_tensor, split_check
+from paper_2608_27128_gb300 import synth
+from paper_2608_27128_gb300 import twinkv as tk
+
+pytestmark = [pytest.mark.gpu, pytest.mark.slow]
+
+
+def run_full(w, ratio):
+    keys, truths = synth.keys(w)
+    S0 = synth.masks(w, ratio)
+    U, N = S0.shape
+    kt = keys_tensor(keys, w.L, w.H)
+    mt = torch.from_numpy(S0.reshape(w.L, w.H, N)).to(device())
+    bud = torch.from_numpy(S0.sum(1).astype(np.int32)).to(device())
+    out = tk.twinkv_repair(kt, mt, bud, threshold=w.tau, want_all=True)
+    torch.cuda.synchronize()
+    assert tk.twinkv_get_last_error() == tk.OK
+    h = {k: v.cpu().numpy() for k, v in out.items()}
+    for k in ("mask", "score_ret", "twin_ret", "score_all", "twin_all"):
+        h[k] = h[k].reshape(U, N)
+    del kt, mt, out
+    torch.cuda.empty_cache()
+    return keys, truths, S0, h
+
+
+def invariants(S0, h, tau):
+    U, N = S0.shape
+    assert np.all(h["status"] == 0)
+    np.testing.assert_array_equal(h["mask"].sum(1), S0.sum(1))            # |S1| = |S0|
+    prot = np.zeros(N, bool)
+    prot[:synth.N_SINK] = True
+    prot[N - synth.N_RECENT:] = True
+    tau_d = float(np.float32(tau))
+    for u in range(U):
+        m = int(h["nswaps"][u])
+        out_, in_ = h["swaps"][u, :m, 0], h["swaps"][u, :m, 1]
+        assert np.all(S0[u, out_] == 1) and np.all(S0[u, in_] == 0)
+        assert np.all(h["score_ret"][u, out_] >= tau_d) and not np.any(prot[out_])
+        assert np.all(h["score_ret"][u, in_] < tau_d)
+        changed = np.flatnonzero(h["mask"][u] != S0[u])
+        assert changed.size == 2 * m
+        assert np.all(h["score_ret"][u] <= h["score_all"][u])
+        t = h["twin_ret"][u]
+        ok = t >= 0
+        assert np.all(S0[u, t[ok]] == 1)
+        assert np.all(np.abs(t[ok] - np.flatnonzero(ok)) > synth.WINDOW)
+
+
+def planted(truths, h, S0, check_needles=False):
+    for u, t in enumerate(truths):
+        for s, c in t.pairs:
+            if c - s > synth.WINDOW:
+                assert h["twin_all"][u, s] == c and h["twin_all"][u, c] == s
+        if check_needles:
+            ev = t.needles[S0[u, t.needles] == 0]
+            assert ev.size > 0
+            assert np.all(h["score_ret"][u, ev] < 0.85)
+            assert np.all(h["mask"][u, ev] == 1)
+
+
+def full_units(keys, S0, h, units, tau):
+    rep = Report()
+    for u in units:
+        a = oracle.audit(keys[u:u + 1], S0[u:u + 1], window=synth.WINDOW)
+        sim = (lambda uu: (lambda i, j: oracle.sim(keys, uu, i, j)))(u)
+        rep.add(compare_best(h["score_ret"][u], h["twin_ret"][u], a["b_ret"][0],
+                             a["t_ret"][0], a["b_ret2"][0], sim, synth.WINDOW, S0=S0[u]))
+        rep.add(compare_best(h["score_all"][u], h["twin_all"][u], a["b_all"][0],
+                             a["t_all"][0], a["b_all2"][0], sim, synth.WINDOW))
+        r = oracle.repair(a["b_ret"], S0[u:u + 1], tau, budget=S0[u:u + 1].sum(1))
+        rep.add(compare_repair(S0[u], h["mask"][u], h["swaps"][u], int(h["nswaps"][u]),
+                               {k: r[k][0] for k in r}, a["b_ret"][0], tau))
+    return rep
+
+
+@pytest.mark.parametrize("ratio", [0.3, 0.5, 0.7])
+def test_llama_full(ratio):
+    w = synth.get("llama")
+    keys, truths, S0, h = run_full(w, ratio)
+    split_check(h, S0, w.tau, synth.N_SINK, synth.N_RECENT)
+    invariants(S0, h, w.tau)
+    planted(truths, h, S0)
+    rep = full_units(keys, S0, h, [0, 77], w.tau)
+    assert rep.n_fail == 0, rep.notes
+    assert rep.max_dev_same_twin < 1e-9
+
+
+@pytest.mark.parametrize("ratio", [0.3, 0.5, 0.7])
+def test_qwen_full(ratio):
+    w = synth.get("qwen")
+    keys, truths, S0, h = run_full(w, ratio)
+    split_check(h, S0, w.tau, synth.N_SINK, synth.N_RECENT)
+    invariants(S0, h, w.tau)
+    planted(truths, h, S0)
+    rep = full_units(keys, S0, h, [5], w.tau)
+    assert rep.n_fail == 0, rep.notes
+    assert rep.max_dev_same_twin < 1e-9
+
+
+def test_retrieval_full():
+    w = synth.get("retrieval")
+    keys, truths, S0, h = run_full(w, 0.3)
+    split_check(h, S0, w.tau, synth.N_SINK, synth.N_RECENT)
+    invariants(S0, h, w.tau)
+    planted(truths, h, S0, check_needles=True)
+    rep = full_units(keys, S0, h, [3], w.tau)
+    assert rep.n_fail == 0, rep.notes
+    assert rep.max_dev_same_twin < 1e-9
+
+
+def test_long_full_sampled_rows():
+    w = synth.get("long")
+    keys, truths, S0, h = run_full(w, 0.5)
+    split_check(h, S0, w.tau, synth.N_SINK, synth.N_RECENT)
+    invariants(S0, h, w.tau)
+    planted(truths, h, S0)
+    rng = np.random.default_rng(5)
+    rows = np.sort(rng.choice(w.N, size=4096, replace=False))
+    a = oracle.audit(keys, S0, window=synth.WINDOW, rows=rows)
+    rep = Report()
+    for u in range(w.units):
+        sim = (lambda uu: (lambda i, j: oracle.sim(keys, uu, i, j)))(u)
+        rep.add(compare_best(h["score_ret"][u, rows], h["twin_ret"][u, rows], a["b_ret"][u],
+                             a["t_ret"][u], a["b_ret2"][u], sim, synth.WINDOW, rows=rows,
+                             S0=S0[u]))
+        rep.add(compare_best(h["score_all"][u, rows], h["twin_all"][u, rows], a["b_all"][u],
+                             a["t_all"][u], a["b_all2"][u], sim, synth.WINDOW, rows=rows))
+    assert rep.n_fail == 0, rep.notes
+    assert rep.max_dev_same_twin < 1e-9
