@@ -310,7 +310,8 @@ def run_ours(args, w, ratio):
                                   "long loop)",
                      "kernel": "twk audit_kernel", "flops_per_launch": flops,
                      "ms_per_launch": audit_ms_per},
-        "kernel_ms_per_step": {k: (t / max(n, 1)) for k, (n, t) in prof.items()},
+        "kernel_ms_per_step": {k: t / args.steps for k, (n, t) in prof.items()},
+        "kernel_launches_per_step": {k: n / args.steps for k, (n, t) in prof.items()},
         "gpu_launches": launches,
         "e2e": {"value": world * U * N / (e2e_ms * 1e-3), "unit": "keys/s",
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms},

@@ -61,8 +61,8 @@
  * error ~1e-13) and fp64 rounding, so it is symmetric in (i, j) and exactly 1 for a
  * duplicate; orphan/donor decisions and the severity ranking use these fp64 values.
  *
- * Limits: d in {64, 128}; 1 <= N <= 1048576; L*H*N*d < 2^31 elements per tensor
- * coordinate; L*H*(N rounded up to 256, plus 256) < 2^31 rows.
+ * Limits: d in {64, 128}; 1 <= N <= 1048576; L*H <= 65535; L*H*N*d < 2^31 elements
+ * per tensor coordinate; L*H*(N rounded up to 256, plus 256) < 2^31 rows.
  */
 #ifndef TWINKV_H
 #define TWINKV_H

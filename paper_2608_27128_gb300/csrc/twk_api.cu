@@ -2,6 +2,8 @@
 // validation, workspace carving, TMA tensor maps and the launch sequence of the
 // TwinKV audit and repair pass (arXiv 2608.27128, Sec. 3.2 and 3.4).
 #include <cmath>
+#include <cstdio>
+#include <cstdlib>
 #include <cstring>
 #include <mutex>
 #include <vector>
@@ -64,7 +66,14 @@ struct ProfScope {
     }
 };
 
-twinkv_status cuda_status(cudaError_t e) { return e == cudaSuccess ? TWINKV_OK : TWINKV_ERR_CUDA; }
+// A failed CUDA call maps to TWINKV_ERR_CUDA; with TWINKV_DEBUG set in the environment
+// its message also goes to stderr.
+twinkv_status cuda_status(cudaError_t e)
+{
+    if (e == cudaSuccess) return TWINKV_OK;
+    if (std::getenv("TWINKV_DEBUG")) std::fprintf(stderr, "twinkv: %s\n", cudaGetErrorString(e));
+    return TWINKV_ERR_CUDA;
+}
 
 // Current device's cached facts; sets them up on first use (outside stream capture).
 twinkv_status device_info(DeviceInfo** out)
@@ -122,7 +131,7 @@ bool shape_ok(const twinkv_shape& s, bool need_d)
 {
     if (s.L < 1 || s.H < 1 || s.N < 1 || s.N > kMaxN) return false;
     const int64_t U = static_cast<int64_t>(s.L) * s.H;
-    if (U > (1 << 24)) return false;
+    if (U > 65535) return false;                             // units run on grid.y
     if (!need_d) return U * s.N < (1LL << 31);
     if (s.d != 64 && s.d != 128) return false;
     if (s.dtype != TWINKV_BF16 && s.dtype != TWINKV_F32) return false;
@@ -155,7 +164,7 @@ Layout layout(const twinkv_shape& s, int op)
         if (s.dtype == TWINKV_F32) L.keys16 = take(U * N * s.d * 2);
         L.colrinv = take(U * NP * 4);
         L.colpos = take(U * NP * 4);
-        L.norm2 = take(U * N * 8);
+        L.norm2 = take(U * N * 16);
         if (op == TWINKV_OP_REPAIR) {
             L.kp = take(U * NP * s.d * 2);
             L.cnt = take(U * N * 4);
@@ -254,15 +263,15 @@ twinkv_status launch_select(const twinkv_shape& s, const double* b, const uint8_
     return cuda_status(launch_repair(r, st));
 }
 
-twinkv_status run_norm2(const uint16_t* k16, const twinkv_shape& s, double* norm2,
+twinkv_status run_norm2(const uint16_t* k16, const twinkv_shape& s, float4* norms,
                         cudaStream_t st)
 {
     ProfScope p(TWINKV_KERNEL_PREP, st);
     return cuda_status(
-        launch_norm2(k16, static_cast<int64_t>(s.L) * s.H * s.N, s.d, norm2, st));
+        launch_norms(k16, static_cast<int64_t>(s.L) * s.H * s.N, s.d, norms, st));
 }
 
-twinkv_status run_refine(const uint16_t* k16, const twinkv_shape& s, const double* norm2,
+twinkv_status run_refine(const uint16_t* k16, const twinkv_shape& s, const float4* norm2,
                          const int* t0, int* t1, double* b0, double* b1, cudaStream_t st)
 {
     ProfScope p(TWINKV_KERNEL_REFINE, st);
@@ -418,7 +427,7 @@ twinkv_status twinkv_redundancy(const void* keys, twinkv_shape s, int32_t window
     const int64_t NP = column_stride(s.N);
     float* colrinv = at<float>(workspace, L.colrinv);
     int* colpos = at<int>(workspace, L.colpos);
-    double* norm2 = at<double>(workspace, L.norm2);
+    float4* norm2 = at<float4>(workspace, L.norm2);
     {
         ProfScope p(TWINKV_KERNEL_PREP, st);
         if (launch_norms_identity(k16, U, s.N, s.d, NP, colrinv, colpos, st) != cudaSuccess)
@@ -440,6 +449,7 @@ twinkv_status twinkv_redundancy(const void* keys, twinkv_shape s, int32_t window
     a.out_t0 = out_twin;
     a.err = dev->err;
     a.timeout_ns = g_timeout_ns;
+    a.mant_mask = 0xFFFFFF80u;
     if ((r = run_audit(*dev, s, k16, k16, static_cast<int64_t>(U) * s.N, a, st)) != TWINKV_OK)
         return r;
     return run_refine(k16, s, norm2, out_twin, nullptr, out_score, nullptr, st);
@@ -470,7 +480,7 @@ twinkv_status twinkv_repair(const void* keys, twinkv_shape s, const uint8_t* ret
     const int64_t NP = column_stride(s.N);
     float* colrinv = at<float>(workspace, L.colrinv);
     int* colpos = at<int>(workspace, L.colpos);
-    double* norm2 = at<double>(workspace, L.norm2);
+    float4* norm2 = at<float4>(workspace, L.norm2);
     uint16_t* kp = at<uint16_t>(workspace, L.kp);
     int* cnt = at<int>(workspace, L.cnt);
     int* kb = at<int>(workspace, L.kb);
@@ -507,6 +517,7 @@ twinkv_status twinkv_repair(const void* keys, twinkv_shape s, const uint8_t* ret
     a.out_t1 = t1;
     a.err = dev->err;
     a.timeout_ns = g_timeout_ns;
+    a.mant_mask = 0xFFFFFF80u;
     if ((r = run_audit(*dev, s, k16, kp, static_cast<int64_t>(U) * NP, a, st)) != TWINKV_OK)
         return r;
     if ((r = run_refine(k16, s, norm2, t0, t1, bret, out_score_all, st)) != TWINKV_OK)

@@ -6,21 +6,21 @@
 //   Sec. 3.4 Eq. 4   b_i(S0) = max over retained j, -1 if none; and its argmax
 //   (b_i(all))       the same over every j
 //
-// Design (one persistent CTA per SM, 320 threads, warp-specialised):
+// Design (one persistent CTA per SM, 64 + 32 * kEpiWarps threads, warp-specialised):
 //   warp 0      TMA producer: the 128-row A block of keys i (once per work item), then
 //               per 256-column tile the B tile of keys j (in 64-wide K chunks) and the
 //               tile's column metadata (1/||k_j|| and original positions).
 //   warp 1      owns TMEM (512 columns = two 128x256 fp32 accumulators) and issues
 //               tcgen05.mma (M=128, N=256, K=16, bf16 -> fp32) from one thread.
-//   warps 2..9  epilogue: warpgroup h in {0,1} takes columns [128h, 128h+128) of each
-//               tile; a thread owns one row (TMEM lane) and keeps its running maximum.
+//   warps 2..   epilogue: four warps per column group g (kGW columns of each tile); a
+//               thread owns one row (TMEM lane) and keeps its running maximum.
 // Keys enter the tensor cores un-normalised (bf16 products are exact in fp32);
 // 1/||k_j|| is applied per element in fp32.  1/||k_i|| > 0 does not change the argmax
 // over j, so it is never applied: this kernel outputs the twin positions, and the
 // exact similarity of each chosen twin is computed afterwards (twk_refine.cu).
 //
 // Max and argmax in one operation: after scaling, the low 7 mantissa bits of each
-// value are replaced by (127 - c), c the column within the warpgroup's 128 columns;
+// value are replaced by (127 - c), c the column within the warp's column group;
 // a plain fp32 max then returns the largest value (to 2^-16 relative, which decides
 // the argmax only among near-equal candidates) and, among equal truncated values,
 // the lowest column.  Columns to ignore carry NaN (max skips
@@ -32,15 +32,19 @@
 // order), so every tile belongs to exactly one of the two maxima.  The kernel writes
 // both winners; the maximum over all columns is the larger of the two, taken on the
 // exact similarities computed afterwards.
+#include <cfloat>
+
 #include "twk_internal.h"
 #include "twk_ptx.cuh"
 
 namespace twk {
 namespace {
 
-constexpr int kThreads = 320;
+constexpr int kEpiWarps = 8;                  // epilogue warps: 2 per SM sub-partition
+constexpr int kGroups = kEpiWarps / 4;        // column groups per tile
+constexpr int kGW = kBN / kGroups;            // columns per group (a multiple of 32)
+constexpr int kThreads = 64 + 32 * kEpiWarps; // + TMA warp + MMA warp
 constexpr uint32_t kTmemCols = 512;
-constexpr uint32_t kMantMask = 0xFFFFFF80u;
 
 template <int D>
 struct AuditCfg {
@@ -49,13 +53,13 @@ struct AuditCfg {
     static constexpr int A_BYTES = KC * A_CHUNK;
     static constexpr int B_STAGE = kBN * 128;         // 32 KB: one K chunk of a tile
     static constexpr int STAGES = (D == 128) ? 4 : 5;
-    static constexpr int MSLOTS = 6;
+    static constexpr int MSLOTS = 8;
     static constexpr int META = kBN * 8;              // rinv[256] + pos[256]
     static constexpr int OFF_A = 0;
     static constexpr int OFF_B = OFF_A + 2 * A_BYTES;
     static constexpr int OFF_META = OFF_B + STAGES * B_STAGE;
-    static constexpr int OFF_X = OFF_META + MSLOTS * META;   // 2 x 128 rows x 16 B
-    static constexpr int OFF_BAR = OFF_X + 2 * kBM * 16;
+    static constexpr int OFF_X = OFF_META + MSLOTS * META;   // 2 x (groups-1) x 128 x 16 B
+    static constexpr int OFF_BAR = OFF_X + 2 * (kGroups - 1) * kBM * 16;
     static constexpr int NBAR = 2 + 2 + 2 * STAGES + 2 * MSLOTS + 2 + 2 + 2 + 2 + 1;
     static constexpr int OFF_MISC = OFF_BAR + NBAR * 8;
     static constexpr int BYTES = OFF_MISC + 16 + 1024;       // + 1024 for alignment
@@ -68,9 +72,11 @@ __device__ __forceinline__ float fmax3(float a, float b, float c)
     return r;
 }
 
-__device__ __forceinline__ float pack(float v, uint32_t idx)
+// (v with its lowest mantissa bits replaced by idx); mask (0xFFFFFF80) is a kernel
+// argument, held in a register, so that idx can be the instruction's immediate.
+__device__ __forceinline__ float pack(float v, uint32_t idx, uint32_t mask)
 {
-    return __uint_as_float((__float_as_uint(v) & kMantMask) | idx);
+    return __uint_as_float((__float_as_uint(v) & mask) | idx);
 }
 
 __device__ __forceinline__ float nan_f() { return __uint_as_float(0x7FFFFFFFu); }
@@ -88,7 +94,7 @@ __device__ __forceinline__ void reg_fence(uint32_t (&x)[32])
                    "+r"(x[27]), "+r"(x[28]), "+r"(x[29]), "+r"(x[30]), "+r"(x[31]));
 }
 
-// Maximum of 32 packed values as a tree of 3-input maxima (depth 4).
+// Maximum of 32 values as a tree of 3-input maxima (depth 4); NaN entries are skipped.
 __device__ __forceinline__ float tree32(const float (&p)[32])
 {
     float q[11];
@@ -102,10 +108,21 @@ __device__ __forceinline__ float tree32(const float (&p)[32])
     return fmax3(r0, r1, fmaxf(r2, r3));
 }
 
-// 32 columns [c0, c0 + 32) of one row: scale by 1/||k_j||, pack the column, reduce.
+// Running best of one row over one segment: the scaled similarity x_ij / ||k_j|| in
+// fp32 (to 2^-16 relative) and its column.
+struct Best {
+    float v;
+    int col;
+};
+
+// Packed maximum of 32 columns: each scaled value x_ij / ||k_j|| has its 7 lowest
+// mantissa bits replaced by (127 - c), c = c0 + k its column within the group, so the
+// maximum carries the largest value (to 2^-16 relative) and, among values equal at
+// that precision, the lowest column.
 template <bool kMasked>
-__device__ __forceinline__ float fold32(const uint32_t (&x)[32], const float* rinv,
-                                        const int* pos, int c0, int rw, uint32_t w2)
+__device__ __forceinline__ float chunk32(const uint32_t (&x)[32], const float* rinv,
+                                         const int* pos, int rw, uint32_t w2, uint32_t mask,
+                                         int c0)
 {
     float p[32];
 #pragma unroll
@@ -126,36 +143,52 @@ __device__ __forceinline__ float fold32(const uint32_t (&x)[32], const float* ri
             v3 = (static_cast<uint32_t>(q.w - rw) > w2) ? v3 : nan_f();
         }
         const uint32_t i0 = 127u - static_cast<uint32_t>(c0 + k);
-        p[k] = pack(v0, i0);
-        p[k + 1] = pack(v1, i0 - 1u);
-        p[k + 2] = pack(v2, i0 - 2u);
-        p[k + 3] = pack(v3, i0 - 3u);
+        p[k] = pack(v0, i0, mask);
+        p[k + 1] = pack(v1, i0 - 1u, mask);
+        p[k + 2] = pack(v2, i0 - 2u, mask);
+        p[k + 3] = pack(v3, i0 - 3u, mask);
     }
     return tree32(p);
 }
 
-// One warpgroup's 128 columns of the accumulator for this thread's row: the second
-// pair of TMEM loads is in flight while the first pair is reduced.
+// One group's kGW columns of the accumulator for this thread's row folded into the
+// running best (a strictly larger maximum replaces it, so an earlier column keeps a
+// tie); the next pair of TMEM loads is in flight while the previous pair is reduced.
 template <bool kMasked>
-__device__ __forceinline__ float half_tile(uint32_t taddr, const float* rinv, const int* pos,
-                                           int rw, uint32_t w2)
+__device__ __forceinline__ void group_tile(uint32_t taddr, const float* rinv, const int* pos,
+                                           int rw, uint32_t w2, uint32_t mask, int col0,
+                                           Best& b)
 {
-    uint32_t x0[32], x1[32], x2[32], x3[32];
+    static_assert(kGW == 64 || kGW == 128, "column group of 64 or 128");
+    uint32_t x0[32], x1[32];
     tmem_ld_32x32b_x32(taddr, x0);
     tmem_ld_32x32b_x32(taddr + 32, x1);
     tmem_wait_ld();
     reg_fence(x0);
     reg_fence(x1);
-    tmem_ld_32x32b_x32(taddr + 64, x2);
-    tmem_ld_32x32b_x32(taddr + 96, x3);
-    const float m0 = fold32<kMasked>(x0, rinv, pos, 0, rw, w2);
-    const float m1 = fold32<kMasked>(x1, rinv + 32, pos + 32, 32, rw, w2);
-    tmem_wait_ld();
-    reg_fence(x2);
-    reg_fence(x3);
-    const float m2 = fold32<kMasked>(x2, rinv + 64, pos + 64, 64, rw, w2);
-    const float m3 = fold32<kMasked>(x3, rinv + 96, pos + 96, 96, rw, w2);
-    return fmax3(m0, m1, fmaxf(m2, m3));
+    float m;
+    if (kGW == 64) {
+        m = fmaxf(chunk32<kMasked>(x0, rinv, pos, rw, w2, mask, 0),
+                  chunk32<kMasked>(x1, rinv + 32, pos + 32, rw, w2, mask, 32));
+    } else {
+        uint32_t x2[32], x3[32];
+        tmem_ld_32x32b_x32(taddr + 64, x2);
+        tmem_ld_32x32b_x32(taddr + 96, x3);
+        const float m0 = chunk32<kMasked>(x0, rinv, pos, rw, w2, mask, 0);
+        const float m1 = chunk32<kMasked>(x1, rinv + 32, pos + 32, rw, w2, mask, 32);
+        tmem_wait_ld();
+        reg_fence(x2);
+        reg_fence(x3);
+        const float m2 = chunk32<kMasked>(x2, rinv + 64, pos + 64, rw, w2, mask, 64);
+        const float m3 = chunk32<kMasked>(x3, rinv + 96, pos + 96, rw, w2, mask, 96);
+        m = fmax3(m0, m1, fmaxf(m2, m3));
+    }
+    const uint32_t mb = __float_as_uint(m);
+    const float tv = __uint_as_float(mb & mask);
+    if (tv > b.v) {
+        b.v = tv;
+        b.col = col0 + 127 - static_cast<int>(mb & 127u);
+    }
 }
 
 struct Tiles {
@@ -192,7 +225,7 @@ __device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity, uint6
 {
     const uint32_t a = smem_u32(bar);
     const uint64_t t0 = globaltimer_ns();
-    while (!mbar_try_wait(a, parity))
+    while (!mbar_try_wait_sleep(a, parity, 1000000u))
         if (globaltimer_ns() - t0 > limit_ns) return;
 }
 
@@ -205,6 +238,8 @@ __device__ __forceinline__ int last_parity(long long total, int n, int s)
     return static_cast<int>((k / n) & 1);
 }
 
+// Registers are per sub-partition (16384 each): with W warps a sub-partition holds
+// ceil(W / 4) of them, which bounds the registers per thread.
 template <int D>
 __global__ void __launch_bounds__(kThreads, 1)
     audit_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
@@ -240,9 +275,9 @@ __global__ void __launch_bounds__(kThreads, 1)
             mbar_init(&a_full[i], 1);
             mbar_init(&a_empty[i], 1);
             mbar_init(&t_full[i], 1);
-            mbar_init(&t_empty[i], 8);
-            mbar_init(&x_full[i], 128);
-            mbar_init(&x_empty[i], 128);
+            mbar_init(&t_empty[i], kEpiWarps);
+            mbar_init(&x_full[i], (kGroups - 1) * kBM);
+            mbar_init(&x_empty[i], kBM);
         }
         for (int i = 0; i < C::STAGES; ++i) {
             mbar_init(&b_full[i], 1);
@@ -250,7 +285,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         for (int i = 0; i < C::MSLOTS; ++i) {
             mbar_init(&m_full[i], 1);
-            mbar_init(&m_empty[i], 8);
+            mbar_init(&m_empty[i], kEpiWarps);
         }
         mbar_init(drain, 1);
         *abort_flag = 0;
@@ -399,13 +434,16 @@ __global__ void __launch_bounds__(kThreads, 1)
     } else {
         // ------------------------------------------------------------ epilogue
         const int ew = warp - 2;
-        const int h = ew >> 2;            // column half of the tile
+        const int h = ew >> 2;            // column group of the tile
         const int q = warp & 3;           // TMEM lane quarter this warp may read
         const int row_local = q * 32 + lane;
         const uint32_t lane_base = static_cast<uint32_t>(q * 32) << 16;
         const int w = a.window;
         const uint32_t w2 = 2u * static_cast<uint32_t>(w);
-        long long n_m = 0, n_t = 0, n_x = 0;
+        const uint32_t mask = a.mant_mask;
+        uint32_t ms = 0, mph = 0;    // meta ring slot and phase
+        uint32_t acc = 0, tph = 0;   // accumulator buffer and phase
+        uint32_t n_x = 0;
         bool ok = true;
         for (int item = blockIdx.x; item < n_items && ok; item += gridDim.x) {
             const int u = item / a.RB;
@@ -435,72 +473,80 @@ __global__ void __launch_bounds__(kThreads, 1)
                 s1b = kpad + hi - chi;
             }
 
-            float bv0 = -INFINITY, bv1 = -INFINITY;   // running best of segment 0 / 1
-            int bc0 = -1, bc1 = -1;                   // and its column
+            Best b0{-INFINITY, -1}, b1{-INFINITY, -1};   // retained (or all) / evicted
             const int rw = row - w;
             for (int t = 0; t < nt; ++t) {
-                const int ms = static_cast<int>(n_m % C::MSLOTS);
-                const int acc = static_cast<int>(n_t & 1);
-                ok = all_wait(&m_full[ms], static_cast<uint32_t>((n_m / C::MSLOTS) & 1), wc, 7);
-                if (ok) ok = all_wait(&t_full[acc], static_cast<uint32_t>((n_t >> 1) & 1), wc, 8);
+                ok = all_wait(&m_full[ms], mph, wc, 7);
+                if (ok) ok = all_wait(&t_full[acc], tph, wc, 8);
                 if (!ok) break;
                 tc_fence_after();
-                const float* rinv = reinterpret_cast<const float*>(sMeta + ms * C::META) + h * kHalf;
+                const float* rinv = reinterpret_cast<const float*>(sMeta + ms * C::META) + h * kGW;
                 const int* pos =
-                    reinterpret_cast<const int*>(sMeta + ms * C::META + kBN * 4) + h * kHalf;
-                const int c_lo = t * kBN + h * kHalf;
-                const bool band = (c_lo < s0b && c_lo + kHalf > s0a) ||
-                                  (c_lo < s1b && c_lo + kHalf > s1a);
-                const uint32_t taddr =
-                    tmem + lane_base + static_cast<uint32_t>(acc * kBN + h * kHalf);
-                const float m = band ? half_tile<true>(taddr, rinv, pos, rw, w2)
-                                     : half_tile<false>(taddr, rinv, pos, rw, w2);
+                    reinterpret_cast<const int*>(sMeta + ms * C::META + kBN * 4) + h * kGW;
+                const int c_lo = t * kBN + h * kGW;
+                const bool band = (c_lo < s0b && c_lo + kGW > s0a) ||
+                                  (c_lo < s1b && c_lo + kGW > s1a);
+                const uint32_t taddr = tmem + lane_base + acc * kBN + static_cast<uint32_t>(h * kGW);
+                if (t < ut.tr) {
+                    if (band) group_tile<true>(taddr, rinv, pos, rw, w2, mask, c_lo, b0);
+                    else group_tile<false>(taddr, rinv, pos, rw, w2, mask, c_lo, b0);
+                } else {
+                    if (t == ut.tr) {
+                        // The evicted segment matters only where it reaches the retained
+                        // one: start its running best just below this group's retained
+                        // best (exact similarities decide between the two later; the
+                        // FLT_MIN keeps an exact tie at 0 in play).
+                        b1.v = b0.v - (fabsf(b0.v) * 0x1p-13f + FLT_MIN);
+                    }
+                    if (band) group_tile<true>(taddr, rinv, pos, rw, w2, mask, c_lo, b1);
+                    else group_tile<false>(taddr, rinv, pos, rw, w2, mask, c_lo, b1);
+                }
                 tc_fence_before();
                 __syncwarp();
                 if (lane == 0) {
                     mbar_arrive(&t_empty[acc]);
                     mbar_arrive(&m_empty[ms]);
                 }
-                ++n_m;
-                ++n_t;
-                const float tv = __uint_as_float(__float_as_uint(m) & kMantMask);
-                const int tc = c_lo + 127 - static_cast<int>(__float_as_uint(m) & 127u);
-                if (t < ut.tr) {
-                    if (tv > bv0) {
-                        bv0 = tv;
-                        bc0 = tc;
-                    }
-                } else if (tv > bv1) {
-                    bv1 = tv;
-                    bc1 = tc;
+                if (++ms == C::MSLOTS) {
+                    ms = 0;
+                    mph ^= 1;
                 }
+                acc ^= 1;
+                tph ^= acc == 0 ? 1u : 0u;
             }
             if (!ok) break;
+            const float bv0 = b0.v, bv1 = b1.v;
+            const int bc0 = b0.col, bc1 = b1.col;
 
-            // Merge the two column halves of every row through shared memory.
+            // Merge the column groups of every row through shared memory: groups
+            // 1.. hand their (value, column) pairs to group 0.
             const int xb = static_cast<int>(n_x & 1);
-            float4* X = sX + xb * kBM;
-            if (h == 1) {
-                ok = all_wait(&x_empty[xb], static_cast<uint32_t>(((n_x >> 1) & 1) ^ 1), wc, 9);
+            float4* X = sX + xb * (kGroups - 1) * kBM;
+            if (h != 0) {
+                ok = all_wait(&x_empty[xb], ((n_x >> 1) & 1) ^ 1, wc, 9);
                 if (!ok) break;
-                X[row_local] = make_float4(bv0, __int_as_float(bc0), bv1, __int_as_float(bc1));
+                X[(h - 1) * kBM + row_local] =
+                    make_float4(bv0, __int_as_float(bc0), bv1, __int_as_float(bc1));
                 mbar_arrive(&x_full[xb]);
             } else {
-                ok = all_wait(&x_full[xb], static_cast<uint32_t>((n_x >> 1) & 1), wc, 10);
+                ok = all_wait(&x_full[xb], (n_x >> 1) & 1, wc, 10);
                 if (!ok) break;
-                const float4 o = X[row_local];
-                mbar_arrive(&x_empty[xb]);
-                float v0 = bv0, v1 = bv1;   // truncated values decide only within a half
+                float v0 = bv0, v1 = bv1;
                 int c0 = bc0, c1 = bc1;
-                const int oc0 = __float_as_int(o.y), oc1 = __float_as_int(o.w);
-                if (oc0 >= 0 && (c0 < 0 || o.x > v0 || (o.x == v0 && oc0 < c0))) {
-                    v0 = o.x;
-                    c0 = oc0;
+#pragma unroll
+                for (int g = 1; g < kGroups; ++g) {
+                    const float4 o = X[(g - 1) * kBM + row_local];
+                    const int oc0 = __float_as_int(o.y), oc1 = __float_as_int(o.w);
+                    if (oc0 >= 0 && (c0 < 0 || o.x > v0 || (o.x == v0 && oc0 < c0))) {
+                        v0 = o.x;
+                        c0 = oc0;
+                    }
+                    if (oc1 >= 0 && (c1 < 0 || o.z > v1 || (o.z == v1 && oc1 < c1))) {
+                        v1 = o.z;
+                        c1 = oc1;
+                    }
                 }
-                if (oc1 >= 0 && (c1 < 0 || o.z > v1 || (o.z == v1 && oc1 < c1))) {
-                    v1 = o.z;
-                    c1 = oc1;
-                }
+                mbar_arrive(&x_empty[xb]);
                 if (row < a.N) {
                     const int64_t o_idx = static_cast<int64_t>(u) * a.N + row;
                     const int64_t cbase = static_cast<int64_t>(u) * a.NP;

@@ -10,7 +10,6 @@ namespace twk {
 
 constexpr int kBM = 128;       // rows (keys i) per work item: the UMMA M
 constexpr int kBN = 256;       // columns (keys j) per tile: the UMMA N
-constexpr int kHalf = kBN / 2; // columns per epilogue warpgroup
 
 // Column stride of the per-unit column arrays (a multiple of kBN with room for the
 // padding of both the retained and the evicted segment).
@@ -31,6 +30,9 @@ struct AuditArgs {
                                 //          (repair mode with need_all), -1 if none
     int* err;
     unsigned long long timeout_ns;
+    uint32_t mant_mask;         // 0xFFFFFF80: clears the 7 mantissa bits that carry the
+                                // column; a runtime value, so the compiler keeps it in a
+                                // register and the pack is a single 3-input logic op
 };
 
 struct RepairArgs {
@@ -60,10 +62,11 @@ cudaError_t launch_gather(const uint16_t* keys, const uint8_t* mask, const int* 
                           float* colrinv, int* colpos, cudaStream_t st);
 
 // exact similarity of the chosen twins
-cudaError_t launch_norm2(const uint16_t* keys, int64_t n, int d, double* norm2, cudaStream_t st);
+// norms[r] = {k.k hi, k.k lo, 1/||k|| hi, 1/||k|| lo} (double-float pairs) per key.
+cudaError_t launch_norms(const uint16_t* keys, int64_t n, int d, float4* norms, cudaStream_t st);
 // b0 = sim(i, twin0); with twin1 given (the evicted-segment winner), twin1 is
 // overwritten with the overall winner and b1 (nullable) receives its similarity.
-cudaError_t launch_refine(const uint16_t* keys, int U, int N, int d, const double* norm2,
+cudaError_t launch_refine(const uint16_t* keys, int U, int N, int d, const float4* norms,
                           const int* twin0, int* twin1, double* b0, double* b1,
                           cudaStream_t st);
 

@@ -62,6 +62,23 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity)
     return ok != 0;
 }
 
+// The same, but the thread may stay suspended for up to `hint_ns` while the phase is
+// incomplete (it resumes as soon as the phase completes): a waiting warp then takes
+// no issue slots from the warps that share its sub-partition.
+__device__ __forceinline__ bool mbar_try_wait_sleep(uint32_t bar, uint32_t parity,
+                                                    uint32_t hint_ns)
+{
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity), "r"(hint_ns)
+        : "memory");
+    return ok != 0;
+}
+
 // Everything a bounded wait needs: the time limit, the block's abort flag (shared
 // memory) and the device error word.
 struct WaitCtl {
@@ -90,9 +107,8 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, const 
     if (mbar_try_wait(a, parity)) return true;
     const uint64_t t0 = globaltimer_ns();
     for (;;) {
-#pragma unroll 1
-        for (int k = 0; k < 32; ++k)
-            if (mbar_try_wait(a, parity)) return true;
+        // suspended for up to ~1 ms per attempt, woken when the phase completes
+        if (mbar_try_wait_sleep(a, parity, 1000000u)) return true;
         if (*w.abort_flag) return false;
         if (globaltimer_ns() - t0 > w.limit_ns) {
             record_timeout(w, where);
