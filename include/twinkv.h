@@ -83,7 +83,9 @@ typedef enum {
     TWINKV_ERR_BUDGET = 3,        /* popcount(mask of unit u) != budget[u] */
     TWINKV_ERR_CUDA = 4,          /* a CUDA runtime/driver call failed */
     TWINKV_ERR_TIMEOUT = 5,       /* a device-side wait gave up; outputs are undefined */
-    TWINKV_ERR_WORKSPACE = 6      /* workspace missing, misaligned or too small */
+    TWINKV_ERR_WORKSPACE = 6,     /* workspace missing, misaligned or too small */
+    TWINKV_ERR_TOO_LARGE = 7      /* more than TWINKV_NOALLOC_MAX_POSITIONS positions were
+                                     given to twinkv_repair_select_noalloc */
 } twinkv_status;
 
 typedef enum { TWINKV_BF16 = 0, TWINKV_F32 = 1 } twinkv_dtype;
@@ -181,6 +183,33 @@ twinkv_status twinkv_repair_select(const double* score_ret, twinkv_shape s,
                                    uint8_t* out_mask, int32_t* out_swaps,
                                    int32_t* out_nswaps, int32_t* out_status,
                                    void* workspace, size_t workspace_bytes, void* stream);
+
+/*
+ * twinkv_repair_select for callers that may not allocate device memory: the same
+ * classification, ranking and swap, with the same arguments and outputs, but without a
+ * workspace argument.  The paper has no counterpart to this entry point; it exists for
+ * callers that cannot call cudaMalloc: a plugin inside a serving engine or framework
+ * that owns every device allocation through its own memory pool, or a latency-critical
+ * loop that cannot afford the device-wide synchronization cudaMalloc and cudaFree may
+ * imply.  The sort buffers live in a fixed array of device memory inside this library
+ * (about 6 MiB per GPU that loads it, held until the process exits), so:
+ *   - L*H*N may be at most TWINKV_NOALLOC_MAX_POSITIONS; larger requests return
+ *     TWINKV_ERR_TOO_LARGE and enqueue nothing;
+ *   - every call on a device shares that one array: two calls that may run at the
+ *     same time on the GPU (for example on different streams without ordering between
+ *     them) race and corrupt each other's results; order them on one stream;
+ *   - the first call on each device looks up the array's device address (a host-side
+ *     setup step, done once per device); make that first call before any stream
+ *     capture.
+ * Nothing is allocated, by this call or on its behalf.
+ */
+#define TWINKV_NOALLOC_MAX_POSITIONS 262144
+twinkv_status twinkv_repair_select_noalloc(const double* score_ret, twinkv_shape s,
+                                           const uint8_t* retained_mask, const int32_t* budget,
+                                           float threshold, const twinkv_params* params,
+                                           uint8_t* out_mask, int32_t* out_swaps,
+                                           int32_t* out_nswaps, int32_t* out_status,
+                                           void* stream);
 
 /* Static description of a status code. */
 const char* twinkv_status_string(twinkv_status st);

@@ -280,6 +280,32 @@ twinkv_status run_refine(const uint16_t* k16, const twinkv_shape& s, const float
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; }
 
+// ---- fixed device scratch for twinkv_repair_select_noalloc ------------------------
+// The selection's sort buffers (two 8-byte keys and two 4-byte positions per position,
+// each buffer rounded up to 256 bytes) for up to TWINKV_NOALLOC_MAX_POSITIONS positions.
+// On the host, g_noalloc_scratch only names the symbol; its device address is looked
+// up per device with cudaGetSymbolAddress.
+constexpr size_t kNoAllocBytes = 24u * TWINKV_NOALLOC_MAX_POSITIONS + 4u * 256u;
+__device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocBytes];
+void* g_noalloc_ptr[kMaxDevices];
+
+// Device address of g_noalloc_scratch on the current device (looked up on first use).
+twinkv_status noalloc_scratch(void** out)
+{
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices)
+        return TWINKV_ERR_CUDA;
+    std::lock_guard<std::mutex> lk(g_mu);
+    if (!g_noalloc_ptr[dev]) {
+        void* p = nullptr;
+        const cudaError_t e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+        if (e != cudaSuccess || !p) return cuda_status(e == cudaSuccess ? cudaErrorUnknown : e);
+        g_noalloc_ptr[dev] = p;
+    }
+    *out = g_noalloc_ptr[dev];
+    return TWINKV_OK;
+}
+
 }  // namespace
 }  // namespace twk
 
@@ -322,6 +348,9 @@ const char* twinkv_status_string(twinkv_status st)
     case TWINKV_ERR_CUDA: return "CUDA error";
     case TWINKV_ERR_TIMEOUT: return "a device-side wait timed out";
     case TWINKV_ERR_WORKSPACE: return "workspace missing, misaligned or too small";
+    case TWINKV_ERR_TOO_LARGE:
+        return "L*H*N exceeds TWINKV_NOALLOC_MAX_POSITIONS (the fixed scratch of "
+               "twinkv_repair_select_noalloc)";
     }
     return "unknown status";
 }
@@ -546,6 +575,32 @@ twinkv_status twinkv_repair_select(const double* score_ret, twinkv_shape s,
     if ((r = device_info(&dev)) != TWINKV_OK) return r;
     return launch_select(s, score_ret, retained_mask, budget, threshold, p, out_mask, out_swaps,
                          out_nswaps, out_status, workspace, L, static_cast<cudaStream_t>(stream));
+}
+
+twinkv_status twinkv_repair_select_noalloc(const double* score_ret, twinkv_shape s,
+                                           const uint8_t* retained_mask, const int32_t* budget,
+                                           float threshold, const twinkv_params* params,
+                                           uint8_t* out_mask, int32_t* out_swaps,
+                                           int32_t* out_nswaps, int32_t* out_status,
+                                           void* stream)
+{
+    const twinkv_params p = params ? *params : twinkv_default_params();
+    if (!score_ret || !retained_mask || !out_mask || !out_nswaps || !shape_ok(s, false) ||
+        (!out_swaps && s.N >= 2))
+        return TWINKV_ERR_INVALID_ARG;
+    twinkv_status r = params_ok(p, threshold);
+    if (r != TWINKV_OK) return r;
+    if (static_cast<int64_t>(s.L) * s.H * s.N > TWINKV_NOALLOC_MAX_POSITIONS)
+        return TWINKV_ERR_TOO_LARGE;
+    const Layout L = layout(s, TWINKV_OP_REPAIR_SELECT);
+    if (L.total > kNoAllocBytes) return TWINKV_ERR_TOO_LARGE;
+    DeviceInfo* dev = nullptr;
+    if ((r = device_info(&dev)) != TWINKV_OK) return r;
+    void* scratch = nullptr;
+    if ((r = noalloc_scratch(&scratch)) != TWINKV_OK) return r;
+    // The sort buffers are fully written before they are read: nothing needs clearing.
+    return launch_select(s, score_ret, retained_mask, budget, threshold, p, out_mask, out_swaps,
+                         out_nswaps, out_status, scratch, L, static_cast<cudaStream_t>(stream));
 }
 
 }  // extern "C"

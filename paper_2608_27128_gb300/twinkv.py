@@ -18,7 +18,9 @@ import torch
 
 from . import build as _build
 
-OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_BUDGET, ERR_CUDA, ERR_TIMEOUT, ERR_WORKSPACE = range(7)
+(OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_BUDGET, ERR_CUDA, ERR_TIMEOUT, ERR_WORKSPACE,
+ ERR_TOO_LARGE) = range(8)
+NOALLOC_MAX_POSITIONS = 262144
 BF16, F32 = 0, 1
 OP_REDUNDANCY, OP_REPAIR, OP_REPAIR_SELECT = 0, 1, 2
 KERNEL_PREP, KERNEL_AUDIT, KERNEL_REPAIR, KERNEL_REFINE = 0, 1, 2, 3
@@ -29,6 +31,7 @@ EXPORTED = (
     "twinkv_workspace_size", "twinkv_redundancy", "twinkv_repair", "twinkv_repair_select",
     "twinkv_status_string", "twinkv_get_last_error", "twinkv_set_wait_timeout_ns",
     "twinkv_wait_probe", "twinkv_profile_begin", "twinkv_profile_end",
+    "twinkv_repair_select_noalloc",
 )
 
 
@@ -84,6 +87,9 @@ def load(build_if_missing: bool = True):
         lib.twinkv_repair_select.argtypes = [_P, Shape, _P, _P, ctypes.c_float,
                                              ctypes.POINTER(Params), _P, _P, _P, _P, _P,
                                              ctypes.c_size_t, _P]
+        lib.twinkv_repair_select_noalloc.argtypes = [_P, Shape, _P, _P, ctypes.c_float,
+                                                     ctypes.POINTER(Params), _P, _P, _P, _P,
+                                                     _P]
         lib.twinkv_status_string.argtypes = [ctypes.c_int]
         lib.twinkv_status_string.restype = ctypes.c_char_p
         lib.twinkv_set_wait_timeout_ns.argtypes = [ctypes.c_uint64]
@@ -91,6 +97,7 @@ def load(build_if_missing: bool = True):
         lib.twinkv_profile_end.argtypes = [ctypes.POINTER(ctypes.c_int32),
                                            ctypes.POINTER(ctypes.c_double)]
         for name in ("twinkv_redundancy", "twinkv_repair", "twinkv_repair_select",
+                     "twinkv_repair_select_noalloc",
                      "twinkv_get_last_error", "twinkv_set_wait_timeout_ns",
                      "twinkv_wait_probe", "twinkv_profile_begin", "twinkv_profile_end"):
             getattr(lib, name).restype = ctypes.c_int
@@ -281,6 +288,39 @@ def twinkv_repair_select(score_ret, retained_mask, budget=None, threshold=None, 
         ctypes.byref(p), _ptr(o["mask"]), _ptr(o["swaps"]), _ptr(o["nswaps"]),
         _ptr(o["status"]), _ptr(ws), ws.numel(), _stream(stream))
     _check(st, "twinkv_repair_select")
+    return o
+
+
+def twinkv_repair_select_noalloc(score_ret, retained_mask, budget=None, threshold=None,
+                                 params=None, *, n_sink=None, n_recent=None, out=None,
+                                 stream=None) -> dict:
+    """twinkv_repair_select without a workspace, for callers that may not allocate
+    device memory: the library's own fixed scratch array holds the sort buffers, so at
+    most NOALLOC_MAX_POSITIONS positions (L*H*N) per call, and calls that may run
+    concurrently on the GPU must be ordered on one stream.  Output tensors are created
+    here when ``out`` does not supply them; pass them in ``out`` to allocate nothing."""
+    if score_ret.dim() != 3:
+        raise ValueError("score_ret must be [L, H, N]")
+    L, H, N = (int(x) for x in score_ret.shape)
+    dev = score_ret.device
+    _need(score_ret, "score_ret", torch.float64, (L, H, N), dev)
+    _need(retained_mask, "retained_mask", torch.uint8, (L, H, N), dev)
+    if budget is not None:
+        _need(budget, "budget", torch.int32, (L * H,), dev)
+    s = Shape(L, H, N, 64, BF16)
+    p = _params(params, threshold, None, n_sink, n_recent)
+    out = dict(out or {})
+    o = {
+        "mask": _out(out.get("mask"), "mask", torch.uint8, (L, H, N), dev),
+        "swaps": _out(out.get("swaps"), "swaps", torch.int32, (L * H, N // 2, 2), dev),
+        "nswaps": _out(out.get("nswaps"), "nswaps", torch.int32, (L * H,), dev),
+        "status": _out(out.get("status"), "status", torch.int32, (L * H,), dev),
+    }
+    st = load().twinkv_repair_select_noalloc(
+        _ptr(score_ret), s, _ptr(retained_mask), _ptr(budget), ctypes.c_float(p.threshold),
+        ctypes.byref(p), _ptr(o["mask"]), _ptr(o["swaps"]), _ptr(o["nswaps"]),
+        _ptr(o["status"]), _stream(stream))
+    _check(st, "twinkv_repair_select_noalloc")
     return o
 
 

@@ -54,7 +54,7 @@ def test_defaults_and_sizes(lib):
 
 
 def test_status_strings(lib):
-    for st in range(7):
+    for st in range(8):
         assert tk.status_string(st)
     assert "unknown" in tk.status_string(99)
 
