@@ -125,14 +125,20 @@ def dist_setup():
     return world, rank, local
 
 
-def max_over_ranks(x: float, world: int) -> float:
+def max_over_ranks(x: float, world: int, device: str = "cuda") -> float:
+    """The largest x over all ranks (the slowest rank's step time)."""
     if world == 1:
         return x
     import torch
     import torch.distributed as dist
-    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    t = torch.tensor([x], dtype=torch.float64, device=device)
     dist.all_reduce(t, op=dist.ReduceOp.MAX)
     return float(t.item())
+
+
+def job_throughput(world: int, keys_per_rank: int, ms_max: float) -> float:
+    """Keys every rank audited in one step, divided by the slowest rank's step time."""
+    return world * keys_per_rank / (ms_max * 1e-3)
 
 
 def barrier(world):
@@ -236,7 +242,7 @@ def run_ours(args, w, ratio):
     barrier(world)
     ms = max_over_ranks(e0.elapsed_time(e1) / args.steps, world)
     assert tk.twinkv_get_last_error() == tk.OK
-    value = world * U * N / (ms * 1e-3)
+    value = job_throughput(world, U * N, ms)
 
     # ---- end to end: pinned host inputs -> device, the call, results -> host
     keys_p = keys_h.pin_memory()
@@ -313,7 +319,7 @@ def run_ours(args, w, ratio):
         "kernel_ms_per_step": {k: t / args.steps for k, (n, t) in prof.items()},
         "kernel_launches_per_step": {k: n / args.steps for k, (n, t) in prof.items()},
         "gpu_launches": launches,
-        "e2e": {"value": world * U * N / (e2e_ms * 1e-3), "unit": "keys/s",
+        "e2e": {"value": job_throughput(world, U * N, e2e_ms), "unit": "keys/s",
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms},
         "clocks": clocks.summary(),
     }

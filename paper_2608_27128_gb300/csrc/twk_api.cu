@@ -263,14 +263,6 @@ twinkv_status launch_select(const twinkv_shape& s, const double* b, const uint8_
     return cuda_status(launch_repair(r, st));
 }
 
-twinkv_status run_norm2(const uint16_t* k16, const twinkv_shape& s, float4* norms,
-                        cudaStream_t st)
-{
-    ProfScope p(TWINKV_KERNEL_PREP, st);
-    return cuda_status(
-        launch_norms(k16, static_cast<int64_t>(s.L) * s.H * s.N, s.d, norms, st));
-}
-
 twinkv_status run_refine(const uint16_t* k16, const twinkv_shape& s, const float4* norm2,
                          const int* t0, int* t1, double* b0, double* b1, cudaStream_t st)
 {
@@ -459,10 +451,10 @@ twinkv_status twinkv_redundancy(const void* keys, twinkv_shape s, int32_t window
     float4* norm2 = at<float4>(workspace, L.norm2);
     {
         ProfScope p(TWINKV_KERNEL_PREP, st);
-        if (launch_norms_identity(k16, U, s.N, s.d, NP, colrinv, colpos, st) != cudaSuccess)
+        if (launch_norms_identity(k16, U, s.N, s.d, NP, colrinv, colpos, norm2, st) !=
+            cudaSuccess)
             return TWINKV_ERR_CUDA;
     }
-    if ((r = run_norm2(k16, s, norm2, st)) != TWINKV_OK) return r;
     AuditArgs a;
     std::memset(&a, 0, sizeof a);
     a.U = U;
@@ -520,10 +512,9 @@ twinkv_status twinkv_repair(const void* keys, twinkv_shape s, const uint8_t* ret
     {
         ProfScope pr(TWINKV_KERNEL_PREP, st);
         if (launch_gather(k16, retained_mask, cnt, kb, U, s.N, s.d, NP, kp, colrinv, colpos,
-                          st) != cudaSuccess)
+                          norm2, st) != cudaSuccess)
             return TWINKV_ERR_CUDA;
     }
-    if ((r = run_norm2(k16, s, norm2, st)) != TWINKV_OK) return r;
     const bool need_all = out_score_all || out_twin_all;
     int* t0 = out_twin_ret ? out_twin_ret : at<int>(workspace, L.twin0);
     int* t1 = need_all ? (out_twin_all ? out_twin_all : at<int>(workspace, L.twin1)) : nullptr;

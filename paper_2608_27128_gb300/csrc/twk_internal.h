@@ -54,16 +54,17 @@ struct RepairArgs {
 
 // prep kernels
 cudaError_t launch_round_bf16(const float* in, uint16_t* out, int64_t n, cudaStream_t st);
+// NP must be a multiple of 64 (column_stride gives a multiple of 256).
 cudaError_t launch_norms_identity(const uint16_t* keys, int U, int N, int d, int64_t NP,
-                                  float* colrinv, int* colpos, cudaStream_t st);
+                                  float* colrinv, int* colpos, float4* norms, cudaStream_t st);
 cudaError_t launch_scan(const uint8_t* mask, int U, int N, int* cnt, int* kb, cudaStream_t st);
 cudaError_t launch_gather(const uint16_t* keys, const uint8_t* mask, const int* cnt,
                           const int* kb, int U, int N, int d, int64_t NP, uint16_t* kp,
-                          float* colrinv, int* colpos, cudaStream_t st);
+                          float* colrinv, int* colpos, float4* norms, cudaStream_t st);
 
 // exact similarity of the chosen twins
-// norms[r] = {k.k hi, k.k lo, 1/||k|| hi, 1/||k|| lo} (double-float pairs) per key.
-cudaError_t launch_norms(const uint16_t* keys, int64_t n, int d, float4* norms, cudaStream_t st);
+// norms[r] = {k.k hi, k.k lo, 1/||k|| hi, 1/||k|| lo} (double-float pairs) per key, as
+// written by the prep kernels.
 // b0 = sim(i, twin0); with twin1 given (the evicted-segment winner), twin1 is
 // overwritten with the overall winner and b1 (nullable) receives its similarity.
 cudaError_t launch_refine(const uint16_t* keys, int U, int N, int d, const float4* norms,

@@ -1,13 +1,14 @@
 // twk_prep.cu -- O(N d) preparation for the audit (TwinKV, arXiv 2608.27128):
 //   * float32 keys -> bf16 (round to nearest even),
-//   * 1/||k|| per key, the l2 normalisation of Sec. 3.2 Eq. 1, applied later as a scale
-//     (a zero key gets 0, so it has similarity 0 with every key),
+//   * per key k . k and 1/||k|| (the l2 normalisation of Sec. 3.2 Eq. 1, applied later
+//     as a scale; a zero key gets 0, so it has similarity 0 with every key),
 //   * the retained-first column layout used by the repair audit: retained keys in
 //     position order, padded to a 256-column tile, then evicted keys in position order,
 //     with per-column 1/||k|| (NaN on padding columns, which the audit then ignores)
 //     and per-column original position.
 #include <cuda_bf16.h>
 
+#include "twk_df.cuh"
 #include "twk_internal.h"
 
 namespace twk {
@@ -24,47 +25,40 @@ __global__ void round_bf16_kernel(const float* __restrict__ in, uint16_t* __rest
         out[i] = __bfloat16_as_ushort(__float2bfloat16_rn(in[i]));
 }
 
-// Sum of squares of one bf16 key row by a full warp; returns 1/||k|| (0 for k = 0).
+constexpr int kPrepThreads = 256;
+constexpr int kKeysPerBlock = kPrepThreads / kParts;   // NP is a multiple of this
+
+// The norm record of one key, computed by its kParts-lane group: k.k and 1/||k|| as
+// double-floats (for the exact similarity values) and 1/||k|| in fp32 (for the audit).
 template <int D>
-__device__ __forceinline__ float warp_rinv(const uint16_t* row, uint32_t (&v)[D / 64])
+__device__ __forceinline__ float4 key_norms(const uint16_t* key, int part, float& rinv32)
 {
-    float sq = 0.f;
-    const uint32_t* r32 = reinterpret_cast<const uint32_t*>(row);
-#pragma unroll
-    for (int k = 0; k < D / 64; ++k) {
-        v[k] = r32[k * 32 + (threadIdx.x & 31)];
-        const float lo = __uint_as_float(v[k] << 16);
-        const float hi = __uint_as_float(v[k] & 0xFFFF0000u);
-        sq = fmaf(lo, lo, sq);
-        sq = fmaf(hi, hi, sq);
-    }
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) sq += __shfl_xor_sync(0xFFFFFFFFu, sq, o);
-    return sq > 0.f ? 1.0f / sqrtf(sq) : 0.f;
+    const DF sq = group_dot_df<D>(key, key, part);
+    const DF rn = sq.h > 0.f ? df_rsqrt(sq) : DF{0.f, 0.f};
+    rinv32 = rn.h;
+    return make_float4(sq.h, sq.l, rn.h, rn.l);
 }
 
-// Mode 0 (keys as given): colrinv[u][p] = 1/||k_p||, colpos[u][p] = p; padding columns
-// p in [N, NP) get NaN / -1.  One warp per column.
+// Mode 0 (keys as given): per column p of unit blockIdx.y, colrinv = 1/||k_p|| and
+// colpos = p, NaN / -1 on the padding columns [N, NP); norms[u][p] = the norm record.
+// Grid (NP / kKeysPerBlock, U), kParts lanes per column.
 template <int D>
-__global__ void norms_identity_kernel(const uint16_t* __restrict__ keys, int U, int N,
-                                      int64_t NP, float* __restrict__ colrinv,
-                                      int* __restrict__ colpos)
+__global__ void __launch_bounds__(kPrepThreads)
+    norms_identity_kernel(const uint16_t* __restrict__ keys, int N, int64_t NP,
+                          float* __restrict__ colrinv, int* __restrict__ colpos,
+                          float4* __restrict__ norms)
 {
-    const int64_t total = static_cast<int64_t>(U) * NP;
-    const int64_t wstride = static_cast<int64_t>(gridDim.x) * (blockDim.x >> 5);
-    for (int64_t c = blockIdx.x * static_cast<int64_t>(blockDim.x >> 5) + (threadIdx.x >> 5);
-         c < total; c += wstride) {
-        const int64_t u = c / NP;
-        const int p = static_cast<int>(c - u * NP);
-        float r = nan_f();
-        if (p < N) {
-            uint32_t v[D / 64];
-            r = warp_rinv<D>(keys + (u * N + p) * D, v);
-        }
-        if ((threadIdx.x & 31) == 0) {
-            colrinv[c] = r;
-            colpos[c] = p < N ? p : -1;
-        }
+    const int part = threadIdx.x % kParts;
+    const int p = blockIdx.x * kKeysPerBlock + threadIdx.x / kParts;
+    const int64_t u = blockIdx.y;
+    // every lane takes part in the shuffles of group_dot_df: padding columns use key 0
+    const int pk = p < N ? p : 0;
+    float r32;
+    const float4 nr = key_norms<D>(keys + (u * N + pk) * D, part, r32);
+    if (part == 0) {
+        colrinv[u * NP + p] = p < N ? r32 : nan_f();
+        colpos[u * NP + p] = p < N ? p : -1;
+        if (p < N) norms[u * N + p] = nr;
     }
 }
 
@@ -111,58 +105,47 @@ __global__ void scan_kernel(const uint8_t* __restrict__ mask, int N, int* __rest
     if (threadIdx.x == 0) kb[u] = carry;
 }
 
-// Mode 1, step 2: one warp per position p of unit u copies key p to its column of the
-// retained-first layout and records 1/||k_p||; one warp per padding column writes NaN.
+// Mode 1, step 2: slot p < N of unit blockIdx.y is key p: its kParts-lane group copies
+// it to its column of the retained-first layout (retained keys in position order, then
+// from the next tile boundary the evicted ones), with 1/||k_p|| (fp32) and p as column
+// metadata, and writes its norm record.  Slots p >= N are the padding columns
+// [K, Kpad) and [Kpad + N - K, NP): zero keys, NaN, -1.  Grid (NP / kKeysPerBlock, U).
 template <int D>
-__global__ void gather_kernel(const uint16_t* __restrict__ keys, const uint8_t* __restrict__ mask,
-                              const int* __restrict__ cnt, const int* __restrict__ kb, int U,
-                              int N, int64_t NP, uint16_t* __restrict__ kp,
-                              float* __restrict__ colrinv, int* __restrict__ colpos)
+__global__ void __launch_bounds__(kPrepThreads)
+    gather_kernel(const uint16_t* __restrict__ keys, const uint8_t* __restrict__ mask,
+                  const int* __restrict__ cnt, const int* __restrict__ kb, int N, int64_t NP,
+                  uint16_t* __restrict__ kp, float* __restrict__ colrinv,
+                  int* __restrict__ colpos, float4* __restrict__ norms)
 {
-    const int64_t total = static_cast<int64_t>(U) * NP;   // N positions + NP-N padding per unit
-    const int64_t wstride = static_cast<int64_t>(gridDim.x) * (blockDim.x >> 5);
-    const int lane = threadIdx.x & 31;
-    for (int64_t g = blockIdx.x * static_cast<int64_t>(blockDim.x >> 5) + (threadIdx.x >> 5);
-         g < total; g += wstride) {
-        const int64_t u = g / NP;
-        const int p = static_cast<int>(g - u * NP);
-        const int k = kb[u];
-        const int kpad = ((k + kBN - 1) / kBN) * kBN;
-        uint32_t* dst32;
-        if (p < N) {
-            const int before = cnt[u * N + p];
-            const int col = mask[u * N + p] ? before : kpad + (p - before);
-            uint32_t v[D / 64];
-            const float r = warp_rinv<D>(keys + (u * N + p) * D, v);
-            dst32 = reinterpret_cast<uint32_t*>(kp + (u * NP + col) * D);
+    constexpr int Q = D / 8 / kParts;   // 16-byte chunks per lane
+    const int part = threadIdx.x % kParts;
+    const int p = blockIdx.x * kKeysPerBlock + threadIdx.x / kParts;
+    const int64_t u = blockIdx.y;
+    const int k = kb[u];
+    const int kpad = ((k + kBN - 1) / kBN) * kBN;
+    const int pk = p < N ? p : 0;   // every lane takes part in the shuffles
+    const uint16_t* key = keys + (u * N + pk) * D;
+    float r32;
+    const float4 nr = key_norms<D>(key, part, r32);
+    int col;
+    if (p < N) {
+        const int before = cnt[u * N + p];
+        col = mask[u * N + p] ? before : kpad + (p - before);
+    } else {
+        const int r = p - N;
+        col = r < kpad - k ? k + r : kpad + (N - k) + (r - (kpad - k));
+    }
+    const uint4* src = reinterpret_cast<const uint4*>(key) + part * Q;
+    uint4* dst = reinterpret_cast<uint4*>(kp + (u * NP + col) * D) + part * Q;
 #pragma unroll
-            for (int t = 0; t < D / 64; ++t) dst32[t * 32 + lane] = v[t];
-            if (lane == 0) {
-                colrinv[u * NP + col] = r;
-                colpos[u * NP + col] = p;
-            }
-        } else {
-            // padding columns: [k, kpad) and [kpad + N - k, NP)
-            const int r = p - N;
-            const int col = r < kpad - k ? k + r : kpad + (N - k) + (r - (kpad - k));
-            dst32 = reinterpret_cast<uint32_t*>(kp + (u * NP + col) * D);
-#pragma unroll
-            for (int t = 0; t < D / 64; ++t) dst32[t * 32 + lane] = 0u;
-            if (lane == 0) {
-                colrinv[u * NP + col] = nan_f();
-                colpos[u * NP + col] = -1;
-            }
-        }
+    for (int q = 0; q < Q; ++q) dst[q] = p < N ? __ldg(src + q) : make_uint4(0u, 0u, 0u, 0u);
+    if (part == 0) {
+        colrinv[u * NP + col] = p < N ? r32 : nan_f();
+        colpos[u * NP + col] = p < N ? p : -1;
+        if (p < N) norms[u * N + p] = nr;
     }
 }
 
-int grid_for(int64_t warps, int per_block_warps)
-{
-    int64_t blocks = (warps + per_block_warps - 1) / per_block_warps;
-    if (blocks > 65535LL * 16) blocks = 65535LL * 16;
-    if (blocks < 1) blocks = 1;
-    return static_cast<int>(blocks);
-}
 
 }  // namespace
 
@@ -176,13 +159,13 @@ cudaError_t launch_round_bf16(const float* in, uint16_t* out, int64_t n, cudaStr
 }
 
 cudaError_t launch_norms_identity(const uint16_t* keys, int U, int N, int d, int64_t NP,
-                                  float* colrinv, int* colpos, cudaStream_t st)
+                                  float* colrinv, int* colpos, float4* norms, cudaStream_t st)
 {
-    const int grid = grid_for(static_cast<int64_t>(U) * NP, 8);
+    const dim3 grid(static_cast<unsigned>(NP / kKeysPerBlock), U);
     if (d == 128)
-        norms_identity_kernel<128><<<grid, 256, 0, st>>>(keys, U, N, NP, colrinv, colpos);
+        norms_identity_kernel<128><<<grid, kPrepThreads, 0, st>>>(keys, N, NP, colrinv, colpos, norms);
     else
-        norms_identity_kernel<64><<<grid, 256, 0, st>>>(keys, U, N, NP, colrinv, colpos);
+        norms_identity_kernel<64><<<grid, kPrepThreads, 0, st>>>(keys, N, NP, colrinv, colpos, norms);
     return cudaGetLastError();
 }
 
@@ -194,15 +177,15 @@ cudaError_t launch_scan(const uint8_t* mask, int U, int N, int* cnt, int* kb, cu
 
 cudaError_t launch_gather(const uint16_t* keys, const uint8_t* mask, const int* cnt,
                           const int* kb, int U, int N, int d, int64_t NP, uint16_t* kp,
-                          float* colrinv, int* colpos, cudaStream_t st)
+                          float* colrinv, int* colpos, float4* norms, cudaStream_t st)
 {
-    const int grid = grid_for(static_cast<int64_t>(U) * NP, 8);
+    const dim3 grid(static_cast<unsigned>(NP / kKeysPerBlock), U);
     if (d == 128)
-        gather_kernel<128><<<grid, 256, 0, st>>>(keys, mask, cnt, kb, U, N, NP, kp, colrinv,
-                                                 colpos);
+        gather_kernel<128><<<grid, kPrepThreads, 0, st>>>(keys, mask, cnt, kb, N, NP, kp,
+                                                           colrinv, colpos, norms);
     else
-        gather_kernel<64><<<grid, 256, 0, st>>>(keys, mask, cnt, kb, U, N, NP, kp, colrinv,
-                                                colpos);
+        gather_kernel<64><<<grid, kPrepThreads, 0, st>>>(keys, mask, cnt, kb, N, NP, kp,
+                                                          colrinv, colpos, norms);
     return cudaGetLastError();
 }
 

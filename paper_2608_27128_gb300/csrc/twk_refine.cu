@@ -15,142 +15,11 @@
 // (norms included) use the same routine and term order, and the product of the two
 // inverse norms is formed symmetrically, so the result is symmetric in (i, j) bit for
 // bit and exactly 1 for a duplicate.
+#include "twk_df.cuh"
 #include "twk_internal.h"
 
 namespace twk {
 namespace {
-
-__device__ __forceinline__ void two_sum_acc(float& hi, float& lo, float p)
-{
-    const float s = __fadd_rn(hi, p);
-    const float bp = __fsub_rn(s, hi);
-    const float e = __fadd_rn(__fsub_rn(hi, __fsub_rn(s, bp)), __fsub_rn(p, bp));
-    hi = s;
-    lo = __fadd_rn(lo, e);
-}
-
-// An unevaluated sum hi + lo of two floats (a double-float).
-struct DFPair {
-    float h, l;
-};
-
-// (hi, lo) + (hi2, lo2) as a double-float sum.  TwoSum gives the exact rounding error
-// whatever the operand order, so the result does not depend on which side is which.
-__device__ __forceinline__ void df_add(float& hi, float& lo, float hi2, float lo2)
-{
-    const float s = __fadd_rn(hi, hi2);
-    const float bp = __fsub_rn(s, hi);
-    float e = __fadd_rn(__fsub_rn(hi, __fsub_rn(s, bp)), __fsub_rn(hi2, bp));
-    e = __fadd_rn(e, __fadd_rn(lo, lo2));
-    hi = __fadd_rn(s, e);
-    lo = __fsub_rn(e, __fsub_rn(hi, s));
-}
-
-constexpr int kParts = 4;   // threads per dot product, each over a contiguous quarter
-
-// One quarter of a . b for two bf16 rows of length D: terms in increasing t.
-template <int D>
-__device__ __forceinline__ void quarter_dot(const uint16_t* __restrict__ a,
-                                            const uint16_t* __restrict__ b, int part,
-                                            float& hi, float& lo)
-{
-    constexpr int Q = D / 8 / kParts;   // 16-byte chunks per quarter
-    const uint4* a4 = reinterpret_cast<const uint4*>(a) + part * Q;
-    const uint4* b4 = reinterpret_cast<const uint4*>(b) + part * Q;
-    hi = 0.f;
-    lo = 0.f;
-#pragma unroll
-    for (int q = 0; q < Q; ++q) {
-        const uint4 va = __ldg(a4 + q);
-        const uint4 vb = __ldg(b4 + q);
-        const uint32_t wa[4] = {va.x, va.y, va.z, va.w};
-        const uint32_t wb[4] = {vb.x, vb.y, vb.z, vb.w};
-#pragma unroll
-        for (int k = 0; k < 4; ++k) {
-            // element 2k (low half) then 2k+1 (high half) of this 16-byte chunk
-            two_sum_acc(hi, lo, __fmul_rn(__uint_as_float(wa[k] << 16), __uint_as_float(wb[k] << 16)));
-            two_sum_acc(hi, lo, __fmul_rn(__uint_as_float(wa[k] & 0xFFFF0000u),
-                                          __uint_as_float(wb[k] & 0xFFFF0000u)));
-        }
-    }
-}
-
-// a . b by the kParts consecutive lanes of a group (every lane passes its part): the
-// quarters are summed as ((q0 + q1) + (q2 + q3)), and every lane of the group returns
-// the same double-float.  All dot products, norms included, go through this routine.
-template <int D>
-__device__ __forceinline__ DFPair group_dot_df(const uint16_t* __restrict__ a,
-                                             const uint16_t* __restrict__ b, int part)
-{
-    float hi, lo;
-    quarter_dot<D>(a, b, part, hi, lo);
-#pragma unroll
-    for (int o = 1; o < kParts; o <<= 1) {
-        const float h2 = __shfl_xor_sync(0xFFFFFFFFu, hi, o);
-        const float l2 = __shfl_xor_sync(0xFFFFFFFFu, lo, o);
-        df_add(hi, lo, h2, l2);
-    }
-    return DFPair{hi, lo};
-}
-
-// ---- double-float (unevaluated fp32 pair) helpers --------------------------------
-
-using DF = DFPair;
-
-// a * b as a double-float.  The cross terms are summed as (a.h * b.l + a.l * b.h), so
-// the result does not depend on the operand order.
-__device__ __forceinline__ DF df_mul(DF a, DF b)
-{
-    const float p = __fmul_rn(a.h, b.h);
-    float e = __fmaf_rn(a.h, b.h, -p);
-    e = __fadd_rn(e, __fadd_rn(__fmul_rn(a.h, b.l), __fmul_rn(a.l, b.h)));
-    const float h = __fadd_rn(p, e);
-    return DF{h, __fsub_rn(e, __fsub_rn(h, p))};
-}
-
-// 1/sqrt(s) for s > 0 (about 2^-44 relative): one Newton step around rsqrtf, with the
-// residual 1 - s r^2 formed in double-float.
-__device__ __forceinline__ DF df_rsqrt(DF s)
-{
-    const float r = rsqrtf(s.h);
-    const float r2h = __fmul_rn(r, r);
-    const float r2l = __fmaf_rn(r, r, -r2h);
-    const float th = __fmul_rn(s.h, r2h);
-    const float tl = __fadd_rn(__fmaf_rn(s.h, r2h, -th),
-                               __fadd_rn(__fmul_rn(s.h, r2l), __fmul_rn(s.l, r2h)));
-    const float e = __fsub_rn(__fsub_rn(1.0f, th), tl);   // 1 - th is exact (th ~ 1)
-    const float c = __fmul_rn(__fmul_rn(r, e), 0.5f);
-    const float h = __fadd_rn(r, c);
-    return DF{h, __fsub_rn(c, __fsub_rn(h, r))};
-}
-
-__device__ __forceinline__ double df_to_double(DF a)
-{
-    return static_cast<double>(a.h) + static_cast<double>(a.l);
-}
-
-// Per key: its squared norm k . k and 1/||k||, both as double-floats, in one float4
-// {k.k hi, k.k lo, rinv hi, rinv lo}; kParts threads per key.
-template <int D>
-__global__ void norms_kernel(const uint16_t* __restrict__ keys, int64_t n,
-                             float4* __restrict__ norms)
-{
-    const int part = threadIdx.x % kParts;
-    const int64_t stride = static_cast<int64_t>(gridDim.x) * (blockDim.x / kParts);
-    const int64_t first = blockIdx.x * static_cast<int64_t>(blockDim.x / kParts) + threadIdx.x / kParts;
-    // every group iterates the same number of times, so the shuffles stay converged
-    const int64_t iters = (n + stride - 1) / stride;
-    for (int64_t it = 0; it < iters; ++it) {
-        const int64_t r = first + it * stride;
-        const int64_t rr = r < n ? r : n - 1;
-        const uint16_t* k = keys + rr * D;
-        const DF sq = group_dot_df<D>(k, k, part);
-        if (part == 0 && r < n) {
-            const DF rn = sq.h > 0.f ? df_rsqrt(sq) : DF{0.f, 0.f};
-            norms[r] = make_float4(sq.h, sq.l, rn.h, rn.l);
-        }
-    }
-}
 
 // sim(i, j) of Eq. 1 from the dot product and the two keys' norm records.
 __device__ __forceinline__ double cosine(DF dot, float4 ni, float4 nj)
@@ -214,24 +83,8 @@ __global__ void __launch_bounds__(kRefineThreads)
     }
 }
 
-int blocks_for(int64_t n, int threads)
-{
-    int64_t b = (n + threads - 1) / threads;
-    if (b > 65535LL * 16) b = 65535LL * 16;
-    return static_cast<int>(b < 1 ? 1 : b);
-}
 
 }  // namespace
-
-cudaError_t launch_norms(const uint16_t* keys, int64_t n, int d, float4* norms, cudaStream_t st)
-{
-    const int blocks = blocks_for(n * kParts, 256);
-    if (d == 128)
-        norms_kernel<128><<<blocks, 256, 0, st>>>(keys, n, norms);
-    else
-        norms_kernel<64><<<blocks, 256, 0, st>>>(keys, n, norms);
-    return cudaGetLastError();
-}
 
 cudaError_t launch_refine(const uint16_t* keys, int U, int N, int d, const float4* norms,
                           const int* twin0, int* twin1, double* b0, double* b1,

@@ -1,15 +1,17 @@
 // twk_repair.cu -- budget-exact repair swap of TwinKV (arXiv 2608.27128, Sec. 3.4).
 //
-// One block of 1024 threads per unit (layer, KV head):
+// One block of 512 threads per unit (layer, KV head):
 //   1. validate S0: every mask byte in {0,1}, popcount == budget (when given);
 //   2. classify  orphan = i not in S0 and b_i < tau,
 //                donor  = j in S0, outside [0, n_sink) and [N - n_recent, N), b_j >= tau;
 //   3. compact both lists in position order (warp ballots + a block scan), each entry a
 //      (severity key, position) pair: orphans keyed by b ascending, donors by b
 //      descending, through an order-preserving fp64 -> u64 map (-0 folded into +0);
-//   4. stable LSD radix sort of each list (8-bit digits, warp match + per-warp digit
-//      counts; a digit position shared by every key is skipped), so equal severities
-//      keep position order (lower position first);
+//   4. per list, the m most severe items: a radix select (byte histograms from the top)
+//      finds the cut, an ordered compaction keeps those items in position order, and a
+//      stable LSD radix sort (8-bit digits, warp match + per-warp digit counts; a digit
+//      position shared by every key is skipped) orders them, so equal severities keep
+//      position order (lower position first);
 //   5. m = min(|O|, |D|): S1 = S0 with the first m donors cleared and the first m
 //      orphans set; swaps[k] = (donor k, orphan k).
 // Sort buffers are caller workspace ([U][N] keys and positions, twice).
@@ -18,7 +20,7 @@
 namespace twk {
 namespace {
 
-constexpr int kT = 1024;
+constexpr int kT = 512;   // two blocks per SM: every unit of a prefill in one wave
 constexpr int kW = kT / 32;
 
 __device__ __forceinline__ uint64_t ordered(double b)
@@ -34,6 +36,7 @@ struct Shared {
     int wsum[2][kW];         // block-scan scratch for the two lists
     int red[4];
     int flag;
+    int sel_digit, sel_before, sel_count;
 };
 
 // Block-wide exclusive scan of two 0/1 flags; returns the prefixes and the chunk totals.
@@ -50,7 +53,7 @@ __device__ __forceinline__ void scan2(Shared& s, int fo, int fd, int& po, int& p
     }
     __syncthreads();
     if (wid == 0) {
-        int a = s.wsum[0][lane], b = s.wsum[1][lane];
+        int a = lane < kW ? s.wsum[0][lane] : 0, b = lane < kW ? s.wsum[1][lane] : 0;
 #pragma unroll
         for (int o = 1; o < 32; o <<= 1) {
             const int ya = __shfl_up_sync(0xFFFFFFFFu, a, o);
@@ -60,8 +63,10 @@ __device__ __forceinline__ void scan2(Shared& s, int fo, int fd, int& po, int& p
                 b += yb;
             }
         }
-        s.wsum[0][lane] = a;   // inclusive
-        s.wsum[1][lane] = b;
+        if (lane < kW) {
+            s.wsum[0][lane] = a;   // inclusive
+            s.wsum[1][lane] = b;
+        }
     }
     __syncthreads();
     po = (wid ? s.wsum[0][wid - 1] : 0) + __popc(bo & lt);
@@ -147,6 +152,86 @@ __device__ int radix_sort(Shared& s, uint64_t* k0, int* i0, uint64_t* k1, int* i
     return cur;
 }
 
+// Moves the m smallest of the n (key, position) items in (kin, iin) to (kout, iout),
+// keeping their order (position order), so that ties at the cut go to the lower
+// positions.  The cut is found byte by byte from the top (a radix select: one
+// histogram per byte over the items that still share the selected prefix), stopping
+// early once the whole boundary bucket is selected.  Requires 0 < m <= n.
+__device__ void select_smallest(Shared& s, const uint64_t* kin, const int* iin, uint64_t* kout,
+                                int* iout, int n, int m)
+{
+    const int lane = threadIdx.x & 31;
+    uint64_t prefix = 0, pmask = 0;
+    int need = m;                 // items still to take among those matching the prefix
+    bool whole = false;           // every item matching the prefix is taken
+    for (int shift = 56; shift >= 0 && !whole; shift -= 8) {
+        if (threadIdx.x < 256) s.base[threadIdx.x] = 0;
+        __syncthreads();
+        for (int c0 = 0; c0 < n; c0 += kT) {
+            const int i = c0 + threadIdx.x;
+            int dg = 256;
+            if (i < n) {
+                const uint64_t key = kin[i];
+                if ((key & pmask) == prefix) dg = static_cast<int>((key >> shift) & 255);
+            }
+            const uint32_t peers = __match_any_sync(0xFFFFFFFFu, dg);
+            if (dg < 256 && lane == __ffs(peers) - 1) atomicAdd(&s.base[dg], __popc(peers));
+        }
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            int run = 0, d = 0;
+            for (; d < 255 && run + s.base[d] < need; ++d) run += s.base[d];
+            s.sel_digit = d;
+            s.sel_before = run;
+            s.sel_count = s.base[d];
+        }
+        __syncthreads();
+        need -= s.sel_before;
+        prefix |= static_cast<uint64_t>(s.sel_digit) << shift;
+        pmask |= 255ull << shift;
+        whole = s.sel_count == need;
+        __syncthreads();
+    }
+    // Ordered compaction: items below the prefix, then those equal to it (all of them
+    // when `whole`, else the first `need` in position order).
+    int base = 0, seen_eq = 0;
+    for (int c0 = 0; c0 < n; c0 += kT) {
+        const int i = c0 + threadIdx.x;
+        int fl = 0, fe = 0;
+        uint64_t key = 0;
+        if (i < n) {
+            key = kin[i];
+            const uint64_t km = key & pmask;
+            fl = km < prefix || (whole && km == prefix);
+            fe = !whole && km == prefix;
+        }
+        int pl, pe, tl, te;
+        scan2(s, fl, fe, pl, pe, tl, te);
+        const int k_eq = max(0, min(te, need - seen_eq));   // eq items taken in this chunk
+        if (fl || (fe && pe < k_eq)) {
+            const int dst = base + pl + min(pe, k_eq);
+            kout[dst] = key;
+            iout[dst] = iin[i];
+        }
+        base += tl + k_eq;
+        seen_eq += te;
+    }
+    __syncthreads();
+}
+
+// The m most severe items of one list, in severity order: (key, position) pairs at
+// (k, i) with scratch (kx, ix) of the same extent; returns the position array holding
+// them.
+__device__ const int* most_severe(Shared& s, uint64_t* k, int* i, uint64_t* kx, int* ix, int n,
+                                  int m)
+{
+    if (n > m) {
+        select_smallest(s, k, i, kx, ix, n, m);
+        return radix_sort(s, kx, ix, k, i, m) ? i : ix;
+    }
+    return radix_sort(s, k, i, kx, ix, n) ? ix : i;
+}
+
 __global__ void __launch_bounds__(kT, 1) repair_kernel(const RepairArgs a)
 {
     __shared__ Shared s;
@@ -230,11 +315,9 @@ __global__ void __launch_bounds__(kT, 1) repair_kernel(const RepairArgs a)
     }
     __syncthreads();
 
-    // 4. severity order
-    const int co = radix_sort(s, k0, i0, k1, i1, n_o);
-    const int cd = radix_sort(s, k0 + n_o, i0 + n_o, k1 + n_o, i1 + n_o, n_d);
-    const int* orph = co ? i1 : i0;
-    const int* don = (cd ? i1 : i0) + n_o;
+    // 4. the m most severe orphans and donors, in severity order
+    const int* orph = most_severe(s, k0, i0, k1, i1, n_o, m);
+    const int* don = most_severe(s, k0 + n_o, i0 + n_o, k1 + n_o, i1 + n_o, n_d, m);
     __syncthreads();
 
     // 5. swap
