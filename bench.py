@@ -245,6 +245,20 @@ def run_ours(args, w, ratio):
     value = job_throughput(world, U * N, ms)
 
     # ---- end to end: pinned host inputs -> device, the call, results -> host
+    e2e_ms, h2d, d2h = None, 0, 0
+    if not args.no_e2e:
+        e2e_ms, h2d, d2h = run_e2e(args, world, step, keys, mask, budget, keys_h, mask_h,
+                                   budget_h, out, stream)
+
+    if rank != 0:
+        return
+    _report(args, w, ratio, world, U, N, d, ms, prof, e2e_ms, h2d, d2h, clocks)
+
+
+def run_e2e(args, world, step, keys, mask, budget, keys_h, mask_h, budget_h, out, stream):
+    import torch
+    L, H, N, d = keys.shape
+    U = L * H
     keys_p = keys_h.pin_memory()
     mask_p = mask_h.pin_memory()
     budget_p = budget_h.pin_memory()
@@ -280,10 +294,11 @@ def run_ours(args, w, ratio):
     assert torch.equal(S1_p, out["mask"].cpu())
     h2d = keys_h.numel() * 2 + mask_h.numel() + budget_h.numel() * 4
     d2h = S1_p.numel() + sw_p.numel() * 4 + ns_p.numel() * 4
+    return e2e_ms, h2d, d2h
 
-    if rank != 0:
-        return
 
+def _report(args, w, ratio, world, U, N, d, ms, prof, e2e_ms, h2d, d2h, clocks):
+    value = job_throughput(world, U * N, ms)
     # ---- roofline of the dominant kernel (the fused audit)
     pk, pk_kind = peaks()
     n_audit, audit_ms = prof["audit"]
@@ -292,16 +307,7 @@ def run_ours(args, w, ratio):
     achieved = flops / (audit_ms_per * 1e-3) / 1e12
     peak = pk["bf16_tflops_sustained"]
     launches = sum(n for n, _ in prof.values())
-    traffic = None
-    tfile = os.path.join(ROOT, "profiles", "audit_traffic.json")
-    if os.path.exists(tfile):
-        try:
-            with open(tfile) as f:
-                tinfo = json.load(f)
-            if tinfo.get("workload") == "qwen" and tinfo.get("kernel_rev") == KERNEL_REV:
-                traffic = tinfo.get("bytes_per_launch")
-        except (OSError, ValueError):
-            traffic = None
+    traffic = audit_traffic(U)
 
     line = {
         "metric": METRIC, "value": value, "unit": "keys/s", "n_gpus": world,
@@ -319,8 +325,9 @@ def run_ours(args, w, ratio):
         "kernel_ms_per_step": {k: t / args.steps for k, (n, t) in prof.items()},
         "kernel_launches_per_step": {k: n / args.steps for k, (n, t) in prof.items()},
         "gpu_launches": launches,
-        "e2e": {"value": job_throughput(world, U * N, e2e_ms), "unit": "keys/s",
-                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms},
+        "e2e": None if e2e_ms is None else {
+            "value": job_throughput(world, U * N, e2e_ms), "unit": "keys/s",
+            "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms},
         "clocks": clocks.summary(),
     }
     if not args.no_cpu:
@@ -330,8 +337,32 @@ def run_ours(args, w, ratio):
     print(json.dumps(line), flush=True)
 
 
-# Revision of the audit kernel the committed DRAM-traffic capture refers to.
-KERNEL_REV = "v1"
+AUDIT_SOURCES = ("twk_audit.cu", "twk_ptx.cuh", "twk_internal.h")
+TRAFFIC_FILE = os.path.join(ROOT, "profiles", "audit_kernel_traffic.txt")
+
+
+def audit_source_sha1() -> str:
+    """Hash of the sources the audit kernel is built from."""
+    import hashlib
+    h = hashlib.sha1()
+    for f in AUDIT_SOURCES:
+        with open(os.path.join(ROOT, "paper_2608_27128_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()
+
+
+def audit_traffic(units: int):
+    """DRAM bytes (read + write) of one audit launch over `units` units of the Qwen3-4B
+    shape, from the committed ncu capture, or None when the kernel sources changed
+    since that capture."""
+    try:
+        with open(TRAFFIC_FILE) as f:
+            kv = dict(line.split(":", 1) for line in f if ":" in line and not line.startswith("#"))
+        if kv.get("kernel_source_sha1", "").strip() != audit_source_sha1():
+            return None
+        return float(kv["dram_bytes_per_unit"]) * units
+    except (OSError, KeyError, ValueError):
+        return None
 
 
 def main():
@@ -344,9 +375,12 @@ def main():
     ap.add_argument("--cpu-units", type=int, default=8)
     ap.add_argument("--cpu-rows", type=int, default=16384)
     ap.add_argument("--no-cpu", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--layers", type=int, default=None,
+                    help="fewer layers of the same workload (for profiler captures)")
     args = ap.parse_args()
     from paper_2608_27128_gb300 import synth
-    w = synth.get("qwen")
+    w = synth.get("qwen") if args.layers is None else synth.get("qwen", L=args.layers)
     if args.impl == "reference":
         run_reference(args, w, args.ratio)
     else:
