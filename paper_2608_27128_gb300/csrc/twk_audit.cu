@@ -151,39 +151,36 @@ __device__ __forceinline__ float chunk32(const uint32_t (&x)[32], const float* r
     return tree32(p);
 }
 
-// One group's kGW columns of the accumulator for this thread's row folded into the
-// running best (a strictly larger maximum replaces it, so an earlier column keeps a
-// tie); the next pair of TMEM loads is in flight while the previous pair is reduced.
-template <bool kMasked>
-__device__ __forceinline__ void group_tile(uint32_t taddr, const float* rinv, const int* pos,
-                                           int rw, uint32_t w2, uint32_t mask, int col0,
-                                           Best& b)
+// The thread's kGW accumulator columns of one tile, loaded into registers (after this,
+// the accumulator may be released: the MMA can overwrite it while x is reduced).
+__device__ __forceinline__ void load_group(uint32_t taddr, uint32_t (&x0)[32], uint32_t (&x1)[32],
+                                           uint32_t (&x2)[32], uint32_t (&x3)[32])
 {
-    static_assert(kGW == 64 || kGW == 128, "column group of 64 or 128");
-    uint32_t x0[32], x1[32];
+    static_assert(kGW == 128, "one 128-column group per warp");
     tmem_ld_32x32b_x32(taddr, x0);
     tmem_ld_32x32b_x32(taddr + 32, x1);
+    tmem_ld_32x32b_x32(taddr + 64, x2);
+    tmem_ld_32x32b_x32(taddr + 96, x3);
     tmem_wait_ld();
     reg_fence(x0);
     reg_fence(x1);
-    float m;
-    if (kGW == 64) {
-        m = fmaxf(chunk32<kMasked>(x0, rinv, pos, rw, w2, mask, 0),
-                  chunk32<kMasked>(x1, rinv + 32, pos + 32, rw, w2, mask, 32));
-    } else {
-        uint32_t x2[32], x3[32];
-        tmem_ld_32x32b_x32(taddr + 64, x2);
-        tmem_ld_32x32b_x32(taddr + 96, x3);
-        const float m0 = chunk32<kMasked>(x0, rinv, pos, rw, w2, mask, 0);
-        const float m1 = chunk32<kMasked>(x1, rinv + 32, pos + 32, rw, w2, mask, 32);
-        tmem_wait_ld();
-        reg_fence(x2);
-        reg_fence(x3);
-        const float m2 = chunk32<kMasked>(x2, rinv + 64, pos + 64, rw, w2, mask, 64);
-        const float m3 = chunk32<kMasked>(x3, rinv + 96, pos + 96, rw, w2, mask, 96);
-        m = fmax3(m0, m1, fmaxf(m2, m3));
-    }
-    const uint32_t mb = __float_as_uint(m);
+    reg_fence(x2);
+    reg_fence(x3);
+}
+
+// Folds the loaded group into the running best (a strictly larger maximum replaces
+// it, so an earlier column keeps a tie).
+template <bool kMasked>
+__device__ __forceinline__ void reduce_group(const uint32_t (&x0)[32], const uint32_t (&x1)[32],
+                                             const uint32_t (&x2)[32], const uint32_t (&x3)[32],
+                                             const float* rinv, const int* pos, int rw,
+                                             uint32_t w2, uint32_t mask, int col0, Best& b)
+{
+    const float m0 = chunk32<kMasked>(x0, rinv, pos, rw, w2, mask, 0);
+    const float m1 = chunk32<kMasked>(x1, rinv + 32, pos + 32, rw, w2, mask, 32);
+    const float m2 = chunk32<kMasked>(x2, rinv + 64, pos + 64, rw, w2, mask, 64);
+    const float m3 = chunk32<kMasked>(x3, rinv + 96, pos + 96, rw, w2, mask, 96);
+    const uint32_t mb = __float_as_uint(fmax3(m0, m1, fmaxf(m2, m3)));
     const float tv = __uint_as_float(mb & mask);
     if (tv > b.v) {
         b.v = tv;
@@ -487,9 +484,16 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const bool band = (c_lo < s0b && c_lo + kGW > s0a) ||
                                   (c_lo < s1b && c_lo + kGW > s1a);
                 const uint32_t taddr = tmem + lane_base + acc * kBN + static_cast<uint32_t>(h * kGW);
+                uint32_t x0[32], x1[32], x2[32], x3[32];
+                load_group(taddr, x0, x1, x2, x3);
+                // The tile is in registers: hand the accumulator back to the MMA warp now,
+                // so it can compute the next-but-one tile while this one is reduced.
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&t_empty[acc]);
                 if (t < ut.tr) {
-                    if (band) group_tile<true>(taddr, rinv, pos, rw, w2, mask, c_lo, b0);
-                    else group_tile<false>(taddr, rinv, pos, rw, w2, mask, c_lo, b0);
+                    if (band) reduce_group<true>(x0, x1, x2, x3, rinv, pos, rw, w2, mask, c_lo, b0);
+                    else reduce_group<false>(x0, x1, x2, x3, rinv, pos, rw, w2, mask, c_lo, b0);
                 } else {
                     if (t == ut.tr) {
                         // The evicted segment matters only where it reaches the retained
@@ -498,15 +502,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                         // FLT_MIN keeps an exact tie at 0 in play).
                         b1.v = b0.v - (fabsf(b0.v) * 0x1p-13f + FLT_MIN);
                     }
-                    if (band) group_tile<true>(taddr, rinv, pos, rw, w2, mask, c_lo, b1);
-                    else group_tile<false>(taddr, rinv, pos, rw, w2, mask, c_lo, b1);
+                    if (band) reduce_group<true>(x0, x1, x2, x3, rinv, pos, rw, w2, mask, c_lo, b1);
+                    else reduce_group<false>(x0, x1, x2, x3, rinv, pos, rw, w2, mask, c_lo, b1);
                 }
-                tc_fence_before();
                 __syncwarp();
-                if (lane == 0) {
-                    mbar_arrive(&t_empty[acc]);
-                    mbar_arrive(&m_empty[ms]);
-                }
+                if (lane == 0) mbar_arrive(&m_empty[ms]);
                 if (++ms == C::MSLOTS) {
                     ms = 0;
                     mph ^= 1;
