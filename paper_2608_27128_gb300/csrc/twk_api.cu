@@ -470,7 +470,7 @@ twinkv_status twinkv_redundancy(const void* keys, twinkv_shape s, int32_t window
     a.out_t0 = out_twin;
     a.err = dev->err;
     a.timeout_ns = g_timeout_ns;
-    a.mant_mask = 0xFFFFFF80u;
+    a.mant_mask = 0xFFFFFFE0u;
     if ((r = run_audit(*dev, s, k16, k16, static_cast<int64_t>(U) * s.N, a, st)) != TWINKV_OK)
         return r;
     return run_refine(k16, s, norm2, out_twin, nullptr, out_score, nullptr, st);
@@ -537,7 +537,7 @@ twinkv_status twinkv_repair(const void* keys, twinkv_shape s, const uint8_t* ret
     a.out_t1 = t1;
     a.err = dev->err;
     a.timeout_ns = g_timeout_ns;
-    a.mant_mask = 0xFFFFFF80u;
+    a.mant_mask = 0xFFFFFFE0u;
     if ((r = run_audit(*dev, s, k16, kp, static_cast<int64_t>(U) * NP, a, st)) != TWINKV_OK)
         return r;
     if ((r = run_refine(k16, s, norm2, t0, t1, bret, out_score_all, st)) != TWINKV_OK)

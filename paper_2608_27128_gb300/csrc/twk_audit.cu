@@ -19,11 +19,11 @@
 // over j, so it is never applied: this kernel outputs the twin positions, and the
 // exact similarity of each chosen twin is computed afterwards (twk_refine.cu).
 //
-// Max and argmax in one operation: after scaling, the low 7 mantissa bits of each
-// value are replaced by (127 - c), c the column within the warp's column group;
-// a plain fp32 max then returns the largest value (to 2^-16 relative, which decides
-// the argmax only among near-equal candidates) and, among equal truncated values,
-// the lowest column.  Columns to ignore carry NaN (max skips
+// Max and argmax: each 32-column chunk is scaled and reduced with 3-input maxima.  When
+// a row of the warp improves its best, the chunk's column is resolved by replacing the
+// low 5 mantissa bits of each value with (31 - c) and taking one more maximum, which
+// returns the lowest column among values equal at 2^-18 relative (near-equal candidates
+// only).  Columns to ignore carry NaN (max skips
 // NaN): padding columns have 1/||k_j|| = NaN, and window columns (|i - j| <= w) are
 // set to NaN on the few tiles that intersect the window band of the row block.
 //
@@ -72,7 +72,7 @@ __device__ __forceinline__ float fmax3(float a, float b, float c)
     return r;
 }
 
-// (v with its lowest mantissa bits replaced by idx); mask (0xFFFFFF80) is a kernel
+// (v with its lowest mantissa bits replaced by idx); mask (0xFFFFFFE0) is a kernel
 // argument, held in a register, so that idx can be the instruction's immediate.
 __device__ __forceinline__ float pack(float v, uint32_t idx, uint32_t mask)
 {
@@ -109,22 +109,25 @@ __device__ __forceinline__ float tree32(const float (&p)[32])
 }
 
 // Running best of one row over one segment: the scaled similarity x_ij / ||k_j|| in
-// fp32 (to 2^-16 relative) and its column.
+// fp32 and its column.
 struct Best {
     float v;
     int col;
 };
 
-// Packed maximum of 32 columns: each scaled value x_ij / ||k_j|| has its 7 lowest
-// mantissa bits replaced by (127 - c), c = c0 + k its column within the group, so the
-// maximum carries the largest value (to 2^-16 relative) and, among values equal at
-// that precision, the lowest column.
+// Folds 32 columns [col0, col0 + 32) into the running best.  Each accumulator value is
+// scaled by 1/||k_j|| (NaN where the window drops the column, or where 1/||k_j|| is
+// NaN on padding) and the chunk's maximum is taken.  Only when some row of the warp
+// improves on its best (strictly, so an earlier column keeps a tie) is the column
+// resolved: each value's 5 lowest mantissa bits are replaced by (31 - column) and one
+// more maximum returns the lowest column among the values equal to the maximum at
+// 2^-18 relative.  Most chunks cost one scale and one max tree.
 template <bool kMasked>
-__device__ __forceinline__ float chunk32(const uint32_t (&x)[32], const float* rinv,
-                                         const int* pos, int rw, uint32_t w2, uint32_t mask,
-                                         int c0)
+__device__ __forceinline__ void fold32(const uint32_t (&x)[32], const float* rinv,
+                                       const int* pos, int rw, uint32_t w2, uint32_t mask,
+                                       int col0, Best& b)
 {
-    float p[32];
+    float v[32];
 #pragma unroll
     for (int k = 0; k < 32; k += 4) {
         const float4 r = *reinterpret_cast<const float4*>(rinv + k);
@@ -133,22 +136,31 @@ __device__ __forceinline__ float chunk32(const uint32_t (&x)[32], const float* r
         const float2 p23 = __fmul2_rn(
             make_float2(__uint_as_float(x[k + 2]), __uint_as_float(x[k + 3])),
             make_float2(r.z, r.w));
-        float v0 = p01.x, v1 = p01.y, v2 = p23.x, v3 = p23.y;
+        v[k] = p01.x;
+        v[k + 1] = p01.y;
+        v[k + 2] = p23.x;
+        v[k + 3] = p23.y;
         if (kMasked) {
             // column j is dropped when |pos_j - row| <= w, i.e. (unsigned)(pos_j - (row - w)) <= 2w
             const int4 q = *reinterpret_cast<const int4*>(pos + k);
-            v0 = (static_cast<uint32_t>(q.x - rw) > w2) ? v0 : nan_f();
-            v1 = (static_cast<uint32_t>(q.y - rw) > w2) ? v1 : nan_f();
-            v2 = (static_cast<uint32_t>(q.z - rw) > w2) ? v2 : nan_f();
-            v3 = (static_cast<uint32_t>(q.w - rw) > w2) ? v3 : nan_f();
+            v[k] = (static_cast<uint32_t>(q.x - rw) > w2) ? v[k] : nan_f();
+            v[k + 1] = (static_cast<uint32_t>(q.y - rw) > w2) ? v[k + 1] : nan_f();
+            v[k + 2] = (static_cast<uint32_t>(q.z - rw) > w2) ? v[k + 2] : nan_f();
+            v[k + 3] = (static_cast<uint32_t>(q.w - rw) > w2) ? v[k + 3] : nan_f();
         }
-        const uint32_t i0 = 127u - static_cast<uint32_t>(c0 + k);
-        p[k] = pack(v0, i0, mask);
-        p[k + 1] = pack(v1, i0 - 1u, mask);
-        p[k + 2] = pack(v2, i0 - 2u, mask);
-        p[k + 3] = pack(v3, i0 - 3u, mask);
     }
-    return tree32(p);
+    const float m = tree32(v);
+    const bool up = m > b.v;
+    if (__any_sync(0xFFFFFFFFu, up)) {
+        float p[32];
+#pragma unroll
+        for (int k = 0; k < 32; ++k) p[k] = pack(v[k], 31u - static_cast<uint32_t>(k), mask);
+        const int c = 31 - static_cast<int>(__float_as_uint(tree32(p)) & 31u);
+        if (up) {
+            b.v = m;
+            b.col = col0 + c;
+        }
+    }
 }
 
 // The thread's kGW accumulator columns of one tile, loaded into registers (after this,
@@ -168,24 +180,17 @@ __device__ __forceinline__ void load_group(uint32_t taddr, uint32_t (&x0)[32], u
     reg_fence(x3);
 }
 
-// Folds the loaded group into the running best (a strictly larger maximum replaces
-// it, so an earlier column keeps a tie).
+// Folds the loaded group into the running best, 32 columns at a time in column order.
 template <bool kMasked>
 __device__ __forceinline__ void reduce_group(const uint32_t (&x0)[32], const uint32_t (&x1)[32],
                                              const uint32_t (&x2)[32], const uint32_t (&x3)[32],
                                              const float* rinv, const int* pos, int rw,
                                              uint32_t w2, uint32_t mask, int col0, Best& b)
 {
-    const float m0 = chunk32<kMasked>(x0, rinv, pos, rw, w2, mask, 0);
-    const float m1 = chunk32<kMasked>(x1, rinv + 32, pos + 32, rw, w2, mask, 32);
-    const float m2 = chunk32<kMasked>(x2, rinv + 64, pos + 64, rw, w2, mask, 64);
-    const float m3 = chunk32<kMasked>(x3, rinv + 96, pos + 96, rw, w2, mask, 96);
-    const uint32_t mb = __float_as_uint(fmax3(m0, m1, fmaxf(m2, m3)));
-    const float tv = __uint_as_float(mb & mask);
-    if (tv > b.v) {
-        b.v = tv;
-        b.col = col0 + 127 - static_cast<int>(mb & 127u);
-    }
+    fold32<kMasked>(x0, rinv, pos, rw, w2, mask, col0, b);
+    fold32<kMasked>(x1, rinv + 32, pos + 32, rw, w2, mask, col0 + 32, b);
+    fold32<kMasked>(x2, rinv + 64, pos + 64, rw, w2, mask, col0 + 64, b);
+    fold32<kMasked>(x3, rinv + 96, pos + 96, rw, w2, mask, col0 + 96, b);
 }
 
 struct Tiles {

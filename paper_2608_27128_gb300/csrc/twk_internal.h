@@ -30,7 +30,7 @@ struct AuditArgs {
                                 //          (repair mode with need_all), -1 if none
     int* err;
     unsigned long long timeout_ns;
-    uint32_t mant_mask;         // 0xFFFFFF80: clears the 7 mantissa bits that carry the
+    uint32_t mant_mask;         // 0xFFFFFFE0: clears the 5 mantissa bits that carry the
                                 // column; a runtime value, so the compiler keeps it in a
                                 // register and the pack is a single 3-input logic op
 };
