@@ -245,38 +245,36 @@ def run_ours(args, w, ratio):
     value = job_throughput(world, U * N, ms)
 
     # ---- end to end: pinned host inputs -> device, the call, results -> host
-    e2e_ms, h2d, d2h = None, 0, 0
+    e2e_ms, h2d, d2h, chunk = None, 0, 0, None
     if not args.no_e2e:
-        e2e_ms, h2d, d2h = run_e2e(args, world, step, keys, mask, budget, keys_h, mask_h,
-                                   budget_h, out, stream)
+        e2e_ms, h2d, d2h, chunk = run_e2e(args, world, w, keys_h, mask_h, budget_h, out, stream)
 
     if rank != 0:
         return
-    _report(args, w, ratio, world, U, N, d, ms, prof, e2e_ms, h2d, d2h, clocks)
+    _report(args, w, ratio, world, U, N, d, ms, prof, e2e_ms, h2d, d2h, chunk, clocks)
 
 
-def run_e2e(args, world, step, keys, mask, budget, keys_h, mask_h, budget_h, out, stream):
+def run_e2e(args, world, w, keys_h, mask_h, budget_h, out, stream):
+    """The same step through the host-buffer entry point: pinned host inputs in, pinned
+    host results out (S1, swap lists and counts, and the audit's b and twin arrays),
+    every copy inside the timed region, overlapped with the computation chunk by chunk."""
     import torch
-    L, H, N, d = keys.shape
+
+    from paper_2608_27128_gb300 import twinkv as tk
+    L, H, N, d = keys_h.shape
     U = L * H
     keys_p = keys_h.pin_memory()
     mask_p = mask_h.pin_memory()
     budget_p = budget_h.pin_memory()
-    S1_p = torch.empty((L, H, N), dtype=torch.uint8).pin_memory()
-    sw_p = torch.empty((U, N // 2, 2), dtype=torch.int32).pin_memory()
-    ns_p = torch.empty((U,), dtype=torch.int32).pin_memory()
-    kd = torch.empty_like(keys)
-    md = torch.empty_like(mask)
-    bd = torch.empty_like(budget)
+    chunk = args.e2e_chunk or max(1, (U + 7) // 8)
+    shape = tk.shape_of(keys_p)
+    arena = tk.host_arena(shape, chunk, device=stream.device)
+    res = None
 
     def e2e_step():
-        kd.copy_(keys_p, non_blocking=True)
-        md.copy_(mask_p, non_blocking=True)
-        bd.copy_(budget_p, non_blocking=True)
-        o = step(kd, md, bd)
-        S1_p.copy_(o["mask"], non_blocking=True)
-        sw_p.copy_(o["swaps"], non_blocking=True)
-        ns_p.copy_(o["nswaps"], non_blocking=True)
+        nonlocal res
+        res = tk.twinkv_repair_host(keys_p, mask_p, budget_p, threshold=w.tau, want_all=True,
+                                    chunk_units=chunk, out=res, arena=arena, stream=stream)
 
     for _ in range(2):
         e2e_step()
@@ -290,14 +288,16 @@ def run_e2e(args, world, step, keys, mask, budget, keys_h, mask_h, budget_h, out
     f1.record(stream)
     torch.cuda.synchronize()
     e2e_ms = max_over_ranks(f0.elapsed_time(f1) / e2e_steps, world)
+    assert tk.twinkv_get_last_error() == tk.OK
     # the step's results match the device-resident run
-    assert torch.equal(S1_p, out["mask"].cpu())
-    h2d = keys_h.numel() * 2 + mask_h.numel() + budget_h.numel() * 4
-    d2h = S1_p.numel() + sw_p.numel() * 4 + ns_p.numel() * 4
-    return e2e_ms, h2d, d2h
+    for k in ("mask", "swaps", "nswaps", "score_all", "twin_ret"):
+        assert torch.equal(res[k], out[k].cpu()), k
+    h2d = keys_p.numel() * keys_p.element_size() + mask_p.numel() + budget_p.numel() * 4
+    d2h = sum(t.numel() * t.element_size() for t in res.values())
+    return e2e_ms, h2d, d2h, chunk
 
 
-def _report(args, w, ratio, world, U, N, d, ms, prof, e2e_ms, h2d, d2h, clocks):
+def _report(args, w, ratio, world, U, N, d, ms, prof, e2e_ms, h2d, d2h, chunk, clocks):
     value = job_throughput(world, U * N, ms)
     # ---- roofline of the dominant kernel (the fused audit)
     pk, pk_kind = peaks()
@@ -327,7 +327,8 @@ def _report(args, w, ratio, world, U, N, d, ms, prof, e2e_ms, h2d, d2h, clocks):
         "gpu_launches": launches,
         "e2e": None if e2e_ms is None else {
             "value": job_throughput(world, U * N, e2e_ms), "unit": "keys/s",
-            "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms},
+            "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms,
+            "api": "twinkv_repair_host", "chunk_units": chunk},
         "clocks": clocks.summary(),
     }
     if not args.no_cpu:
@@ -376,6 +377,8 @@ def main():
     ap.add_argument("--cpu-rows", type=int, default=16384)
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--e2e-chunk", type=int, default=0,
+                    help="units per chunk of the host-buffer call (0: an eighth of L*H)")
     ap.add_argument("--layers", type=int, default=None,
                     help="fewer layers of the same workload (for profiler captures)")
     args = ap.parse_args()

@@ -211,6 +211,31 @@ twinkv_status twinkv_repair_select_noalloc(const double* score_ret, twinkv_shape
                                            int32_t* out_nswaps, int32_t* out_status,
                                            void* stream);
 
+/*
+ * twinkv_repair on a cache held in host memory (for example a KV cache offloaded to the
+ * host): the same audit and swap (Sec. 3.4), with every tensor argument a HOST pointer
+ * of the layout above (page-locked memory lets the copies run asynchronously).  The
+ * units are processed in chunks of `chunk_units` units (0: a quarter of L*H): chunk
+ * c + 1 is copied to the device while chunk c is computed on `stream`, and results are
+ * copied back while later chunks run, so the copies hide behind the computation.
+ *   arena        caller-owned DEVICE memory of twinkv_host_arena_size(s, chunk_units)
+ *                bytes, 256-byte aligned: double-buffered chunk inputs and outputs plus
+ *                one chunk's workspace.  The library allocates nothing.
+ *   out_*        host outputs as in twinkv_repair (out_score_ret .. out_twin_all may be
+ *                NULL); valid once `stream` has completed.
+ * The copies run on two streams the library keeps per device; calls on one device are
+ * ordered after each other's use of the arena.
+ */
+size_t twinkv_host_arena_size(twinkv_shape s, int32_t chunk_units);
+twinkv_status twinkv_repair_host(const void* keys, twinkv_shape s, const uint8_t* retained_mask,
+                                 const int32_t* budget, float threshold,
+                                 const twinkv_params* params, uint8_t* out_mask,
+                                 int32_t* out_swaps, int32_t* out_nswaps, double* out_score_ret,
+                                 int32_t* out_twin_ret, double* out_score_all,
+                                 int32_t* out_twin_all, int32_t* out_status,
+                                 int32_t chunk_units, void* arena, size_t arena_bytes,
+                                 void* stream);
+
 /* Static description of a status code. */
 const char* twinkv_status_string(twinkv_status st);
 

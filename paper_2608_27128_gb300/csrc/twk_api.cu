@@ -21,6 +21,7 @@ constexpr int kMaxDevices = 64;
 constexpr int64_t kMaxN = 1 << 20;
 
 std::mutex g_mu;
+std::mutex g_host_mu;   // orders twinkv_repair_host calls' use of the per-device streams
 unsigned long long g_timeout_ns = 2000000000ull;
 
 struct DeviceInfo {
@@ -271,6 +272,76 @@ twinkv_status run_refine(const uint16_t* k16, const twinkv_shape& s, const float
 }
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; }
+
+// ---- host-buffer pipeline (twinkv_repair_host) ------------------------------------
+int default_chunk_units(int U) { return U < 4 ? U : (U + 3) / 4; }
+
+struct HostArena {
+    size_t keys = 0, mask = 0, budget = 0, omask = 0, oswaps = 0, onswaps = 0, ostatus = 0,
+           osret = 0, otret = 0, osall = 0, otall = 0;
+    size_t per_buf = 0, ws = 0, ws_bytes = 0, total = 0;
+};
+
+// One chunk's inputs and outputs (twice, for double buffering) and one workspace.
+HostArena host_arena(const twinkv_shape& s, int uc)
+{
+    HostArena A;
+    size_t off = 0;
+    auto take = [&](size_t bytes) {
+        const size_t o = off;
+        off += up256(bytes);
+        return o;
+    };
+    const size_t N = static_cast<size_t>(s.N), U = static_cast<size_t>(uc);
+    const size_t esize = s.dtype == TWINKV_F32 ? 4 : 2;
+    A.keys = take(U * N * s.d * esize);
+    A.mask = take(U * N);
+    A.budget = take(U * 4);
+    A.omask = take(U * N);
+    A.oswaps = take(U * (N / 2) * 2 * 4);
+    A.onswaps = take(U * 4);
+    A.ostatus = take(U * 4);
+    A.osret = take(U * N * 8);
+    A.otret = take(U * N * 4);
+    A.osall = take(U * N * 8);
+    A.otall = take(U * N * 4);
+    A.per_buf = off;
+    twinkv_shape sc = s;
+    sc.L = 1;
+    sc.H = uc;
+    A.ws = 2 * A.per_buf;
+    A.ws_bytes = layout(sc, TWINKV_OP_REPAIR).total;
+    A.total = A.ws + A.ws_bytes;
+    return A;
+}
+
+struct HostStreams {
+    bool ready = false;
+    cudaStream_t h2d = nullptr, d2h = nullptr;
+    cudaEvent_t in[2], done[2], out[2];
+};
+HostStreams g_hs[kMaxDevices];
+
+twinkv_status host_streams(HostStreams** out)
+{
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices)
+        return TWINKV_ERR_CUDA;
+    HostStreams& h = g_hs[dev];
+    if (!h.ready) {
+        if (cudaStreamCreateWithFlags(&h.h2d, cudaStreamNonBlocking) != cudaSuccess ||
+            cudaStreamCreateWithFlags(&h.d2h, cudaStreamNonBlocking) != cudaSuccess)
+            return TWINKV_ERR_CUDA;
+        for (int b = 0; b < 2; ++b)
+            if (cudaEventCreateWithFlags(&h.in[b], cudaEventDisableTiming) != cudaSuccess ||
+                cudaEventCreateWithFlags(&h.done[b], cudaEventDisableTiming) != cudaSuccess ||
+                cudaEventCreateWithFlags(&h.out[b], cudaEventDisableTiming) != cudaSuccess)
+                return TWINKV_ERR_CUDA;
+        h.ready = true;
+    }
+    *out = &h;
+    return TWINKV_OK;
+}
 
 // ---- fixed device scratch for twinkv_repair_select_noalloc ------------------------
 // The selection's sort buffers (two 8-byte keys and two 4-byte positions per position,
@@ -592,6 +663,112 @@ twinkv_status twinkv_repair_select_noalloc(const double* score_ret, twinkv_shape
     // The sort buffers are fully written before they are read: nothing needs clearing.
     return launch_select(s, score_ret, retained_mask, budget, threshold, p, out_mask, out_swaps,
                          out_nswaps, out_status, scratch, L, static_cast<cudaStream_t>(stream));
+}
+
+size_t twinkv_host_arena_size(twinkv_shape s, int32_t chunk_units)
+{
+    if (!shape_ok(s, true) || chunk_units < 0) return 0;
+    const int U = s.L * s.H;
+    const int uc = chunk_units == 0 ? default_chunk_units(U) : (chunk_units < U ? chunk_units : U);
+    return host_arena(s, uc).total;
+}
+
+twinkv_status twinkv_repair_host(const void* keys, twinkv_shape s, const uint8_t* retained_mask,
+                                 const int32_t* budget, float threshold,
+                                 const twinkv_params* params, uint8_t* out_mask,
+                                 int32_t* out_swaps, int32_t* out_nswaps, double* out_score_ret,
+                                 int32_t* out_twin_ret, double* out_score_all,
+                                 int32_t* out_twin_all, int32_t* out_status,
+                                 int32_t chunk_units, void* arena, size_t arena_bytes,
+                                 void* stream)
+{
+    const twinkv_params p = params ? *params : twinkv_default_params();
+    if (!keys || !retained_mask || !out_mask || !out_nswaps || !shape_ok(s, true) ||
+        (!out_swaps && s.N >= 2) || chunk_units < 0)
+        return TWINKV_ERR_INVALID_ARG;
+    twinkv_status r = params_ok(p, threshold);
+    if (r != TWINKV_OK) return r;
+    const int U = s.L * s.H;
+    const int uc = chunk_units == 0 ? default_chunk_units(U) : (chunk_units < U ? chunk_units : U);
+    const HostArena A = host_arena(s, uc);
+    if (!arena || (reinterpret_cast<uintptr_t>(arena) & 255) != 0 || arena_bytes < A.total)
+        return TWINKV_ERR_WORKSPACE;
+    DeviceInfo* dev = nullptr;
+    if ((r = device_info(&dev)) != TWINKV_OK) return r;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    std::lock_guard<std::mutex> call_lk(g_host_mu);
+    HostStreams* hs = nullptr;
+    if ((r = host_streams(&hs)) != TWINKV_OK) return r;
+
+    char* base = static_cast<char*>(arena);
+    const size_t N = static_cast<size_t>(s.N);
+    const size_t esize = s.dtype == TWINKV_F32 ? 4 : 2;
+    const size_t swaps_per_unit = (N / 2) * 2;
+    auto ck = [&](cudaError_t e) { return e == cudaSuccess; };
+    // The previous call's last uses of both buffers come first.
+    for (int b = 0; b < 2; ++b) {
+        if (!ck(cudaStreamWaitEvent(hs->h2d, hs->done[b], 0)) ||
+            !ck(cudaStreamWaitEvent(hs->h2d, hs->out[b], 0)) ||
+            !ck(cudaStreamWaitEvent(st, hs->out[b], 0)))
+            return TWINKV_ERR_CUDA;
+    }
+    const int nchunks = (U + uc - 1) / uc;
+    for (int c = 0; c < nchunks; ++c) {
+        const int b = c & 1;
+        const size_t u0 = static_cast<size_t>(c) * uc;
+        const int un = static_cast<int>(U - u0 < static_cast<size_t>(uc) ? U - u0 : uc);
+        char* buf = base + b * A.per_buf;
+        // inputs, once the compute that last read this buffer is done
+        if (c >= 2 && !ck(cudaStreamWaitEvent(hs->h2d, hs->done[b], 0))) return TWINKV_ERR_CUDA;
+        if (!ck(cudaMemcpyAsync(buf + A.keys, static_cast<const char*>(keys) + u0 * N * s.d * esize,
+                                un * N * s.d * esize, cudaMemcpyHostToDevice, hs->h2d)) ||
+            !ck(cudaMemcpyAsync(buf + A.mask, retained_mask + u0 * N, un * N,
+                                cudaMemcpyHostToDevice, hs->h2d)) ||
+            (budget && !ck(cudaMemcpyAsync(buf + A.budget, budget + u0, un * 4,
+                                           cudaMemcpyHostToDevice, hs->h2d))) ||
+            !ck(cudaEventRecord(hs->in[b], hs->h2d)))
+            return TWINKV_ERR_CUDA;
+        // compute on the caller's stream, once the inputs landed and this buffer's
+        // previous outputs were copied out
+        if (!ck(cudaStreamWaitEvent(st, hs->in[b], 0))) return TWINKV_ERR_CUDA;
+        if (c >= 2 && !ck(cudaStreamWaitEvent(st, hs->out[b], 0))) return TWINKV_ERR_CUDA;
+        twinkv_shape sc = s;
+        sc.L = 1;
+        sc.H = un;
+        r = twinkv_repair(buf + A.keys, sc, reinterpret_cast<const uint8_t*>(buf + A.mask),
+                          budget ? reinterpret_cast<const int32_t*>(buf + A.budget) : nullptr,
+                          threshold, &p, reinterpret_cast<uint8_t*>(buf + A.omask),
+                          reinterpret_cast<int32_t*>(buf + A.oswaps),
+                          reinterpret_cast<int32_t*>(buf + A.onswaps),
+                          out_score_ret ? reinterpret_cast<double*>(buf + A.osret) : nullptr,
+                          out_twin_ret ? reinterpret_cast<int32_t*>(buf + A.otret) : nullptr,
+                          out_score_all ? reinterpret_cast<double*>(buf + A.osall) : nullptr,
+                          out_twin_all ? reinterpret_cast<int32_t*>(buf + A.otall) : nullptr,
+                          reinterpret_cast<int32_t*>(buf + A.ostatus), base + A.ws, A.ws_bytes,
+                          st);
+        if (r != TWINKV_OK) return r;
+        if (!ck(cudaEventRecord(hs->done[b], st))) return TWINKV_ERR_CUDA;
+        // outputs
+        if (!ck(cudaStreamWaitEvent(hs->d2h, hs->done[b], 0))) return TWINKV_ERR_CUDA;
+        auto d2h = [&](void* dst, size_t off, size_t bytes) {
+            return ck(cudaMemcpyAsync(dst, buf + off, bytes, cudaMemcpyDeviceToHost, hs->d2h));
+        };
+        if (!d2h(out_mask + u0 * N, A.omask, un * N) ||
+            (out_swaps && !d2h(out_swaps + u0 * swaps_per_unit, A.oswaps,
+                               un * swaps_per_unit * 4)) ||
+            !d2h(out_nswaps + u0, A.onswaps, un * 4) ||
+            (out_status && !d2h(out_status + u0, A.ostatus, un * 4)) ||
+            (out_score_ret && !d2h(out_score_ret + u0 * N, A.osret, un * N * 8)) ||
+            (out_twin_ret && !d2h(out_twin_ret + u0 * N, A.otret, un * N * 4)) ||
+            (out_score_all && !d2h(out_score_all + u0 * N, A.osall, un * N * 8)) ||
+            (out_twin_all && !d2h(out_twin_all + u0 * N, A.otall, un * N * 4)) ||
+            !ck(cudaEventRecord(hs->out[b], hs->d2h)))
+            return TWINKV_ERR_CUDA;
+    }
+    // The caller's stream completes only after the last results reached the host.
+    for (int b = 0; b < 2; ++b)
+        if (!ck(cudaStreamWaitEvent(st, hs->out[b], 0))) return TWINKV_ERR_CUDA;
+    return TWINKV_OK;
 }
 
 }  // extern "C"

@@ -31,7 +31,7 @@ EXPORTED = (
     "twinkv_workspace_size", "twinkv_redundancy", "twinkv_repair", "twinkv_repair_select",
     "twinkv_status_string", "twinkv_get_last_error", "twinkv_set_wait_timeout_ns",
     "twinkv_wait_probe", "twinkv_profile_begin", "twinkv_profile_end",
-    "twinkv_repair_select_noalloc",
+    "twinkv_repair_select_noalloc", "twinkv_host_arena_size", "twinkv_repair_host",
 )
 
 
@@ -90,6 +90,11 @@ def load(build_if_missing: bool = True):
         lib.twinkv_repair_select_noalloc.argtypes = [_P, Shape, _P, _P, ctypes.c_float,
                                                      ctypes.POINTER(Params), _P, _P, _P, _P,
                                                      _P]
+        lib.twinkv_host_arena_size.argtypes = [Shape, ctypes.c_int32]
+        lib.twinkv_host_arena_size.restype = ctypes.c_size_t
+        lib.twinkv_repair_host.argtypes = [_P, Shape, _P, _P, ctypes.c_float,
+                                           ctypes.POINTER(Params), _P, _P, _P, _P, _P, _P, _P,
+                                           _P, ctypes.c_int32, _P, ctypes.c_size_t, _P]
         lib.twinkv_status_string.argtypes = [ctypes.c_int]
         lib.twinkv_status_string.restype = ctypes.c_char_p
         lib.twinkv_set_wait_timeout_ns.argtypes = [ctypes.c_uint64]
@@ -97,7 +102,7 @@ def load(build_if_missing: bool = True):
         lib.twinkv_profile_end.argtypes = [ctypes.POINTER(ctypes.c_int32),
                                            ctypes.POINTER(ctypes.c_double)]
         for name in ("twinkv_redundancy", "twinkv_repair", "twinkv_repair_select",
-                     "twinkv_repair_select_noalloc",
+                     "twinkv_repair_select_noalloc", "twinkv_repair_host",
                      "twinkv_get_last_error", "twinkv_set_wait_timeout_ns",
                      "twinkv_wait_probe", "twinkv_profile_begin", "twinkv_profile_end"):
             getattr(lib, name).restype = ctypes.c_int
@@ -321,6 +326,103 @@ def twinkv_repair_select_noalloc(score_ret, retained_mask, budget=None, threshol
         ctypes.byref(p), _ptr(o["mask"]), _ptr(o["swaps"]), _ptr(o["nswaps"]),
         _ptr(o["status"]), _stream(stream))
     _check(st, "twinkv_repair_select_noalloc")
+    return o
+
+
+def _need_host(t, name, dtype, shape):
+    if not isinstance(t, torch.Tensor):
+        raise TypeError(f"{name} must be a torch tensor")
+    if t.device.type != "cpu":
+        raise ValueError(f"{name} must be a host tensor")
+    if t.dtype != dtype:
+        raise ValueError(f"{name} must be {dtype}, got {t.dtype}")
+    if tuple(t.shape) != tuple(shape):
+        raise ValueError(f"{name} must have shape {tuple(shape)}, got {tuple(t.shape)}")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    return t
+
+
+def _out_host(t, name, dtype, shape, pin):
+    if t is None:
+        return torch.empty(shape, dtype=dtype, pin_memory=pin)
+    return _need_host(t, name, dtype, shape)
+
+
+def twinkv_host_arena_size(shape: Shape, chunk_units: int = 0) -> int:
+    return int(load().twinkv_host_arena_size(shape, int(chunk_units)))
+
+
+def host_arena(shape: Shape, chunk_units: int = 0, device=None) -> torch.Tensor:
+    """A device arena for twinkv_repair_host (torch's allocator: 512-byte aligned)."""
+    n = twinkv_host_arena_size(shape, chunk_units)
+    if n == 0:
+        raise ValueError("invalid shape or chunk size")
+    return torch.empty(n, dtype=torch.uint8, device=device or torch.cuda.current_device())
+
+
+_arenas = {}
+
+
+def _cached_arena(shape: Shape, chunk_units: int) -> torch.Tensor:
+    """The binding's own arena for the current device, grown on demand.  It stays alive
+    between calls because the library's copy streams may still be using it when a call
+    returns; the library orders successive calls' use of it."""
+    dev = torch.cuda.current_device()
+    n = twinkv_host_arena_size(shape, chunk_units)
+    if n == 0:
+        raise ValueError("invalid shape or chunk size")
+    a = _arenas.get(dev)
+    if a is None or a.numel() < n:
+        if a is not None:
+            torch.cuda.synchronize(dev)   # the old arena may still be in use
+        a = _arenas[dev] = torch.empty(n, dtype=torch.uint8, device=dev)
+    return a
+
+
+def twinkv_repair_host(keys, retained_mask, budget=None, threshold=None, params=None, *,
+                       window=None, n_sink=None, n_recent=None, want_ret=True, want_all=False,
+                       chunk_units=0, out=None, arena=None, stream=None) -> dict:
+    """twinkv_repair on HOST tensors (a cache held in host memory): the units go to the
+    device in chunks whose copies overlap the computation of other chunks.  Inputs and
+    the returned outputs are CPU tensors (pinned ones copy asynchronously); the outputs
+    are valid once ``stream`` (default: the current stream) has completed.  ``arena`` is
+    a device uint8 tensor of twinkv_host_arena_size bytes that the caller keeps alive
+    until the stream has completed (a cached one of the binding's when not given)."""
+    s = shape_of(keys)
+    _need_host(keys, "keys", keys.dtype, keys.shape)
+    L, H, N = s.L, s.H, s.N
+    _need_host(retained_mask, "retained_mask", torch.uint8, (L, H, N))
+    if budget is not None:
+        _need_host(budget, "budget", torch.int32, (L * H,))
+    p = _params(params, threshold, window, n_sink, n_recent)
+    pin = keys.is_pinned()
+    out = dict(out or {})
+    o = {
+        "mask": _out_host(out.get("mask"), "mask", torch.uint8, (L, H, N), pin),
+        "swaps": _out_host(out.get("swaps"), "swaps", torch.int32, (L * H, N // 2, 2), pin),
+        "nswaps": _out_host(out.get("nswaps"), "nswaps", torch.int32, (L * H,), pin),
+        "status": _out_host(out.get("status"), "status", torch.int32, (L * H,), pin),
+    }
+    if want_ret:
+        o["score_ret"] = _out_host(out.get("score_ret"), "score_ret", torch.float64,
+                                   (L, H, N), pin)
+        o["twin_ret"] = _out_host(out.get("twin_ret"), "twin_ret", torch.int32, (L, H, N), pin)
+    if want_all:
+        o["score_all"] = _out_host(out.get("score_all"), "score_all", torch.float64,
+                                   (L, H, N), pin)
+        o["twin_all"] = _out_host(out.get("twin_all"), "twin_all", torch.int32, (L, H, N), pin)
+    if arena is None:
+        arena = _cached_arena(s, chunk_units)
+    if not arena.is_cuda or arena.dtype != torch.uint8:
+        raise ValueError("arena must be a CUDA uint8 tensor")
+    st = load().twinkv_repair_host(
+        _ptr(keys), s, _ptr(retained_mask), _ptr(budget), ctypes.c_float(p.threshold),
+        ctypes.byref(p), _ptr(o["mask"]), _ptr(o["swaps"]), _ptr(o["nswaps"]),
+        _ptr(o.get("score_ret")), _ptr(o.get("twin_ret")), _ptr(o.get("score_all")),
+        _ptr(o.get("twin_all")), _ptr(o["status"]), int(chunk_units), _ptr(arena),
+        arena.numel(), _stream(stream))
+    _check(st, "twinkv_repair_host")
     return o
 
 
