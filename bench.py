@@ -290,8 +290,11 @@ def run_e2e(args, world, w, keys_h, mask_h, budget_h, out, stream):
     e2e_ms = max_over_ranks(f0.elapsed_time(f1) / e2e_steps, world)
     assert tk.twinkv_get_last_error() == tk.OK
     # the step's results match the device-resident run
-    for k in ("mask", "swaps", "nswaps", "score_all", "twin_ret"):
+    for k in ("mask", "nswaps", "score_all", "twin_ret"):
         assert torch.equal(res[k], out[k].cpu()), k
+    sw = out["swaps"].cpu()
+    for u, m in enumerate(res["nswaps"].tolist()):
+        assert torch.equal(res["swaps"][u, :max(m, 0)], sw[u, :max(m, 0)]), u
     h2d = keys_p.numel() * keys_p.element_size() + mask_p.numel() + budget_p.numel() * 4
     d2h = sum(t.numel() * t.element_size() for t in res.values())
     return e2e_ms, h2d, d2h, chunk

@@ -222,7 +222,9 @@ twinkv_status twinkv_repair_select_noalloc(const double* score_ret, twinkv_shape
  *                bytes, 256-byte aligned: double-buffered chunk inputs and outputs plus
  *                one chunk's workspace.  The library allocates nothing.
  *   out_*        host outputs as in twinkv_repair (out_score_ret .. out_twin_all may be
- *                NULL); valid once `stream` has completed.
+ *                NULL); valid once `stream` has completed.  Unlike twinkv_repair, the
+ *                entries of out_swaps past out_nswaps[u] are overwritten with
+ *                unspecified values (whole chunks are copied back).
  * The copies run on two streams the library keeps per device; calls on one device are
  * ordered after each other's use of the arena.
  */

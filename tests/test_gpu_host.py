@@ -59,10 +59,14 @@ def _host_run(keys, S0, L, H, tau, want_all, chunk, pin, stream=None):
 
 
 def _assert_same(h, d):
+    """Equal outputs; a unit's swap list is defined up to its nswaps entries only."""
     assert set(h) == set(d)
     for k in d:
         assert h[k].device.type == "cpu"
-        assert torch.equal(h[k], d[k]), k
+        if k != "swaps":
+            assert torch.equal(h[k], d[k]), k
+    for u, m in enumerate(d["nswaps"].tolist()):
+        assert torch.equal(h["swaps"][u, :max(m, 0)], d["swaps"][u, :max(m, 0)]), u
 
 
 @pytest.mark.parametrize("chunk,pin", [(0, True), (1, True), (4, True), (6, True),
