@@ -51,6 +51,11 @@ def _load():
             lib.twk_oracle_audit.argtypes = [
                 _P, ctypes.c_int, ctypes.c_int, ctypes.c_int, _P, ctypes.c_int, _P,
                 ctypes.c_int, _P, _P, _P, _P, _P, _P]
+            lib.twk_oracle_count.argtypes = [
+                _P, ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_float,
+                ctypes.c_double, _P, ctypes.c_int, _P, _P, _P]
+            lib.twk_oracle_policy_select.argtypes = [
+                ctypes.c_int, ctypes.c_int, _P, ctypes.c_int, ctypes.c_int, _P, _P, _P]
             for name in ("twk_oracle_repair", "twk_oracle_repair_f32"):
                 getattr(lib, name).argtypes = [
                     ctypes.c_int, ctypes.c_int, _P, _P, _P, ctypes.c_float, ctypes.c_int,
@@ -160,3 +165,43 @@ def repair_f32(b_ret, mask, threshold: float, n_sink: int = 4, n_recent: int = 6
     """Selection-only entry: the same repair on float32 b values (e.g. a GPU's own)."""
     return _repair(_load().twk_oracle_repair_f32, b_ret, mask, threshold, n_sink,
                    n_recent, budget, np.float32)
+
+
+def count(keys, threshold: float, window: int = 32, band: float = 0.0, rows=None) -> dict:
+    """Redundancy counts of Eq. 2 per unit and row: r (sim > tau, tau rounded to float),
+    r_lo (sim > tau + band) and r_hi (sim > tau - band), each [U, nrows] int32."""
+    k = _keys3(keys)
+    U, N, d = k.shape
+    r = None
+    nrows = N
+    if rows is not None:
+        r = np.ascontiguousarray(np.asarray(rows, dtype=np.int32).ravel())
+        nrows = r.size
+    out = {n: np.empty((U, nrows), np.int32) for n in ("r", "r_lo", "r_hi")}
+    _load().twk_oracle_count(_ptr(k), U, N, d, int(window), ctypes.c_float(threshold),
+                             float(band), _ptr(r), nrows, _ptr(out["r"]), _ptr(out["r_lo"]),
+                             _ptr(out["r_hi"]))
+    return out
+
+
+def policy_select(r, budget, n_sink: int = 4, n_recent: int = 64) -> dict:
+    """The standalone policy of Sec. 3.2 (Eq. 3) on counts r [U,N]: keep budget[u]
+    positions ordered by (protected, s = -r/N descending, position).  Returns mask
+    [U,N] uint8 and status [U]."""
+    r = np.ascontiguousarray(np.asarray(r, dtype=np.int32))
+    U = r.shape[0] if r.ndim == 2 else 1
+    r = r.reshape(U, -1)
+    N = r.shape[1]
+    bud = np.ascontiguousarray(np.broadcast_to(np.asarray(budget, dtype=np.int32), (U,)))
+    out = {"mask": np.empty((U, N), np.uint8), "status": np.empty(U, np.int32)}
+    _load().twk_oracle_policy_select(U, N, _ptr(r), int(n_sink), int(n_recent), _ptr(bud),
+                                     _ptr(out["mask"]), _ptr(out["status"]))
+    return out
+
+
+def policy(keys, threshold: float, budget, window: int = 32, n_sink: int = 4,
+           n_recent: int = 64) -> dict:
+    """Counts (Eq. 2) and the policy's retained set (Eq. 3) for keys [U,N,d]."""
+    c = count(keys, threshold, window)
+    p = policy_select(c["r"], budget, n_sink, n_recent)
+    return {"r": c["r"], **p}

@@ -25,6 +25,10 @@
  *   Sec. 3.4, repair     rank orphans by ascending b, donors by descending b,
  *                        m = min(|O|,|D|), evict the m most severe donors and admit
  *                        the m most severe orphans; |S1| = |S0|
+ *   Sec. 3.2, Eq. 2      r_i = number of j with |i-j| > w (j != i) and sim(i,j) > tau
+ *   Sec. 3.2, Eq. 3      s_i = -r_i / n; the standalone policy keeps the K highest
+ *                        scores, with the sink and recent regions given the maximum
+ *                        score (always kept)
  *
  * Readings where the paper is silent (each one is listed in the design notes):
  *   - a key with zero norm has khat = 0, so its similarity with every key is 0;
@@ -35,7 +39,10 @@
  *   - threshold comparisons use the threshold rounded to float, widened to double,
  *     so that a float implementation and this oracle compare against the same number;
  *   - keys are bf16 bit patterns; float32 keys are first rounded to bf16,
- *     round-to-nearest-even.
+ *     round-to-nearest-even;
+ *   - the standalone policy orders positions by (protected first, r ascending, i.e.
+ *     s descending, then position ascending) and keeps the first K; a budget below
+ *     the protected count keeps the lowest protected positions.
  *
  * Parity pins for every function here live in tests/test_oracle_pins.py and
  * tests/golden/ (closed forms, hand-derived worked examples, a float64 numpy matmul,
@@ -307,4 +314,98 @@ void twk_oracle_repair_f32(int U, int N, const float* b, const uint8_t* mask,
     twk_oracle_repair(U, N, bd, mask, budget, threshold, n_sink, n_recent, out_mask, swaps,
                       nswaps, status, is_orphan, is_donor);
     free(bd);
+}
+
+/* ---- Sec. 3.2, Eq. 2-3: the standalone redundancy policy ----------------------- */
+
+/*
+ * Redundancy counts of Eq. 2.  For each unit u and requested row i:
+ *   r[i]    = #{ j : |i-j| > w, j != i, sim(i,j) > tau }     (Eq. 2, strict)
+ *   r_lo[i] = the same count with tau + band in place of tau
+ *   r_hi[i] = the same count with tau - band in place of tau
+ * so that r_lo <= r <= r_hi, and a count taken in lower precision lies in
+ * [r_lo, r_hi] whenever its similarity errors stay below band.  tau is the
+ * threshold rounded to float and widened.  rows as in twk_oracle_audit; r_lo and
+ * r_hi may be NULL.  out: [U][nrows].
+ */
+void twk_oracle_count(const uint16_t* keys, int U, int N, int d, int window, float threshold,
+                      double band, const int32_t* rows, int nrows, int32_t* r,
+                      int32_t* r_lo, int32_t* r_hi)
+{
+    const double tau = (double)threshold;
+    if (rows == NULL)
+        nrows = N;
+    double* sq = (double*)malloc(sizeof(double) * (size_t)(N > 0 ? N : 1));
+    for (int u = 0; u < U; ++u) {
+        const uint16_t* K = keys + (long)u * N * d;
+        for (int i = 0; i < N; ++i)
+            sq[i] = dot_bf16(&K[(long)i * d], &K[(long)i * d], d);
+#pragma omp parallel for schedule(dynamic, 8)
+        for (int q = 0; q < nrows; ++q) {
+            int i = rows ? rows[q] : q;
+            int c = 0, c_lo = 0, c_hi = 0;
+            for (int j = 0; j < N; ++j) {
+                int dist = (i > j) ? i - j : j - i;
+                if (j == i || dist <= window)
+                    continue;
+                double s = cosine(dot_bf16(&K[(long)i * d], &K[(long)j * d], d), sq[i], sq[j]);
+                c += s > tau;
+                c_lo += s > tau + band;
+                c_hi += s > tau - band;
+            }
+            long o = (long)u * nrows + q;
+            r[o] = c;
+            if (r_lo) r_lo[o] = c_lo;
+            if (r_hi) r_hi[o] = c_hi;
+        }
+    }
+    free(sq);
+}
+
+typedef struct {
+    int32_t prot;   /* 1 for a sink or recent position */
+    int32_t r;
+    int32_t pos;
+} policy_rank;
+
+/* protected first, then fewer twins (higher s = -r/n), then lower position */
+static int cmp_policy(const void* pa, const void* pb)
+{
+    const policy_rank* a = (const policy_rank*)pa;
+    const policy_rank* b = (const policy_rank*)pb;
+    if (a->prot != b->prot) return b->prot - a->prot;
+    if (a->r != b->r) return (a->r > b->r) - (a->r < b->r);
+    return (a->pos > b->pos) - (a->pos < b->pos);
+}
+
+/*
+ * The standalone policy of Sec. 3.2: from the counts r[U][N] (Eq. 2), keep budget[u]
+ * positions of each unit, ordered by (protected first, s = -r/N descending, position
+ * ascending).  Protected: i < n_sink or i >= N - n_recent.  out_mask[U][N] gets 1 for
+ * a kept position.  status[u]: 0 ok, 1 when budget[u] is outside [0, N] (then the
+ * unit's mask is all 0).
+ */
+void twk_oracle_policy_select(int U, int N, const int32_t* r, int n_sink, int n_recent,
+                              const int32_t* budget, uint8_t* out_mask, int32_t* status)
+{
+    policy_rank* e = (policy_rank*)malloc(sizeof(policy_rank) * (size_t)(N > 0 ? N : 1));
+    for (int u = 0; u < U; ++u) {
+        uint8_t* S = out_mask + (long)u * N;
+        memset(S, 0, (size_t)N);
+        const int K = budget[u];
+        if (K < 0 || K > N) {
+            status[u] = 1;
+            continue;
+        }
+        status[u] = 0;
+        for (int i = 0; i < N; ++i) {
+            e[i].prot = (i < n_sink) || (i >= N - n_recent);
+            e[i].r = r[(long)u * N + i];
+            e[i].pos = i;
+        }
+        qsort(e, (size_t)N, sizeof(policy_rank), cmp_policy);
+        for (int k = 0; k < K; ++k)
+            S[e[k].pos] = 1;
+    }
+    free(e);
 }
