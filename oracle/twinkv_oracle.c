@@ -368,13 +368,15 @@ typedef struct {
     int32_t pos;
 } policy_rank;
 
-/* protected first, then fewer twins (higher s = -r/n), then lower position */
+/* Protected positions all carry the maximum score (Sec. 3.2), so they come first and
+ * tie among themselves; unprotected ones follow by fewer twins (higher s = -r/n);
+ * equal scores go by lower position. */
 static int cmp_policy(const void* pa, const void* pb)
 {
     const policy_rank* a = (const policy_rank*)pa;
     const policy_rank* b = (const policy_rank*)pb;
     if (a->prot != b->prot) return b->prot - a->prot;
-    if (a->r != b->r) return (a->r > b->r) - (a->r < b->r);
+    if (!a->prot && a->r != b->r) return (a->r > b->r) - (a->r < b->r);
     return (a->pos > b->pos) - (a->pos < b->pos);
 }
 

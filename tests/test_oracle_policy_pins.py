@@ -124,19 +124,24 @@ def test_count_row_subset_matches_full(oracle_mod):
 
 # ---------------------------------------------------------------- selection (Eq. 3)
 
-@pytest.mark.parametrize("seed", range(10))
+@pytest.mark.parametrize("seed", range(12))
 def test_policy_matches_python_sort(oracle_mod, seed):
-    """Brute force: Python's sorted() on (not protected, r, position), first K kept."""
+    """Brute force from the scores themselves: s_i = -r_i / N (Eq. 3), +inf on the
+    protected regions (their maximum score, Sec. 3.2); Python's sorted() on
+    (-s, position) and the first K kept."""
     rng = np.random.default_rng(seed)
     U = 3
     N = int(rng.integers(1, 300))
     n_sink, n_recent = int(rng.integers(0, 6)), int(rng.integers(0, 20))
+    if seed % 4 == 3:
+        n_recent = N + 3                                    # every position protected
     r = rng.integers(0, 6, size=(U, N)).astype(np.int32)   # many ties
     K = rng.integers(0, N + 1, size=U).astype(np.int32)
     p = oracle_mod.policy_select(r, K, n_sink, n_recent)
     prot = protected(N, n_sink, n_recent)
     for u in range(U):
-        order = sorted(range(N), key=lambda i: (not prot[i], int(r[u, i]), i))
+        score = [float("inf") if prot[i] else -int(r[u, i]) / N for i in range(N)]
+        order = sorted(range(N), key=lambda i: (-score[i], i))
         expect = np.zeros(N, np.uint8)
         expect[order[:K[u]]] = 1
         np.testing.assert_array_equal(p["mask"][u], expect)
@@ -163,7 +168,7 @@ def test_policy_invariants(oracle_mod):
 
 def test_policy_budget_edges(oracle_mod):
     N = 100
-    r = np.arange(N, dtype=np.int32)[None].repeat(5, 0)
+    r = (N - np.arange(N, dtype=np.int32))[None].repeat(5, 0)   # fewer twins later
     K = np.array([0, N, 10, N + 1, -1], np.int32)
     p = oracle_mod.policy_select(r, K, 4, 64)
     assert p["mask"][0].sum() == 0 and p["status"][0] == 0
