@@ -45,9 +45,13 @@ def peaks():
         return dict(FALLBACK), "fallback"
 
 
-def workload_config(w, ratio):
+def workload_config(w, ratio, path="repair"):
+    what = ("audit + repair (Sec. 3.4)" if path == "repair"
+            else "standalone policy: counts + selection (Sec. 3.2 Eq. 2-3)")
     return {
-        "workload": f"Qwen3-4B KV cache {w.L}x{w.H}x{w.N}x{w.d} bf16 (synthetic), ratio {ratio}",
+        "workload": f"Qwen3-4B KV cache {w.L}x{w.H}x{w.N}x{w.d} bf16 (synthetic), ratio {ratio}, "
+                    f"{what}",
+        "path": path,
         "L": w.L, "H": w.H, "N": w.N, "d": w.d, "ratio": ratio, "tau": w.tau,
         "window": 32, "n_sink": 4, "n_recent": 64,
         "budget_per_unit": None,
@@ -147,7 +151,7 @@ def barrier(world):
         dist.barrier()
 
 
-def cpu_sample(w, ratio, units, rows_per_unit):
+def cpu_sample(w, ratio, units, rows_per_unit, path="repair"):
     """Oracle (fp64, host cores) on `units` units, `rows_per_unit` rows each (all columns).
 
     Returns (keys/s, seconds, threads, description)."""
@@ -159,12 +163,19 @@ def cpu_sample(w, ratio, units, rows_per_unit):
     S0 = synth.masks(w, ratio, units=ul)
     rows = np.sort(np.random.default_rng(0).choice(w.N, size=rows_per_unit, replace=False))
     t0 = time.perf_counter()
-    oracle.audit(keys, S0, window=32, rows=rows)
+    if path == "policy":
+        oracle.count(keys, w.tau, window=32, rows=rows)
+    else:
+        oracle.audit(keys, S0, window=32, rows=rows)
     dt = time.perf_counter() - t0
     threads = int(os.environ.get("OMP_NUM_THREADS", os.cpu_count() or 1))
     n = units * rows_per_unit
-    desc = (f"{units} unit(s) x {rows_per_unit} rows (of {w.N}), every column, both maxima; "
-            "the O(N d) repair step is not in the sample")
+    if path == "policy":
+        desc = (f"{units} unit(s) x {rows_per_unit} rows (of {w.N}), every column, the "
+                "Eq. 2 counts; the O(N) selection step is not in the sample")
+    else:
+        desc = (f"{units} unit(s) x {rows_per_unit} rows (of {w.N}), every column, both "
+                "maxima; the O(N d) repair step is not in the sample")
     return n / dt, dt, threads, desc
 
 
@@ -174,7 +185,7 @@ def run_reference(args, w, ratio):
         return
     vals = []
     for _ in range(args.warmup + args.steps):
-        v, dt, threads, desc = cpu_sample(w, ratio, args.cpu_units, args.cpu_rows)
+        v, dt, threads, desc = cpu_sample(w, ratio, args.cpu_units, args.cpu_rows, args.path)
         vals.append((v, dt))
     timed = vals[args.warmup:]
     v = statistics.median(x[0] for x in timed)
@@ -183,7 +194,7 @@ def run_reference(args, w, ratio):
         "metric": METRIC, "value": v, "unit": "keys/s", "n_gpus": args.gpus,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
-        "data": "synthetic", "config": workload_config(w, ratio), "impl": "reference",
+        "data": "synthetic", "config": workload_config(w, ratio, args.path), "impl": "reference",
         "cpu_baseline": {"value": v, "unit": "keys/s", "cores": threads, "kind": "oracle",
                          "sample": desc},
         "e2e": {"value": v, "unit": "keys/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
@@ -216,9 +227,16 @@ def run_ours(args, w, ratio):
     ws = tk.workspace(shape, tk.OP_REPAIR, dev)
     out = None
 
+    if args.path == "policy":
+        ws = tk.workspace(shape, tk.OP_POLICY, dev)
+        K = torch.full((U,), tk.budget_for_ratio(N, ratio), dtype=torch.int32, device=dev)
+
     def step(k=keys, m=mask, b=budget):
         nonlocal out
-        out = tk.twinkv_repair(k, m, b, threshold=w.tau, want_all=True, out=out, ws=ws)
+        if args.path == "policy":
+            out = tk.twinkv_policy(k, K, threshold=w.tau, out=out, ws=ws)
+        else:
+            out = tk.twinkv_repair(k, m, b, threshold=w.tau, want_all=True, out=out, ws=ws)
         return out
 
     for _ in range(args.warmup):
@@ -246,7 +264,7 @@ def run_ours(args, w, ratio):
 
     # ---- end to end: pinned host inputs -> device, the call, results -> host
     e2e_ms, h2d, d2h, chunk = None, 0, 0, None
-    if not args.no_e2e:
+    if not args.no_e2e and args.path == "repair":
         e2e_ms, h2d, d2h, chunk = run_e2e(args, world, w, keys_h, mask_h, budget_h, out, stream)
 
     if rank != 0:
@@ -310,20 +328,22 @@ def _report(args, w, ratio, world, U, N, d, ms, prof, e2e_ms, h2d, d2h, chunk, c
     achieved = flops / (audit_ms_per * 1e-3) / 1e12
     peak = pk["bf16_tflops_sustained"]
     launches = sum(n for n, _ in prof.values())
-    traffic = audit_traffic(U)
+    traffic = audit_traffic(U) if args.path == "repair" else None
 
     line = {
         "metric": METRIC, "value": value, "unit": "keys/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
-        "data": "synthetic", "config": workload_config(w, ratio),
+        "data": "synthetic", "config": workload_config(w, ratio, args.path),
         "tflops_audit": achieved,
         "frac_of_burst_peak": achieved / pk["bf16_tflops"],
         "roofline": {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
                      "frac": achieved / peak, "traffic": traffic,
                      "peak_kind": f"{pk_kind} bf16_tflops_sustained (kernel timed inside a "
                                   "long loop)",
-                     "kernel": "twk audit_kernel", "flops_per_launch": flops,
+                     "kernel": "twk audit_kernel" + (" (count mode)" if args.path == "policy"
+                                                     else ""),
+                     "flops_per_launch": flops,
                      "ms_per_launch": audit_ms_per},
         "kernel_ms_per_step": {k: t / args.steps for k, (n, t) in prof.items()},
         "kernel_launches_per_step": {k: n / args.steps for k, (n, t) in prof.items()},
@@ -335,7 +355,7 @@ def _report(args, w, ratio, world, U, N, d, ms, prof, e2e_ms, h2d, d2h, chunk, c
         "clocks": clocks.summary(),
     }
     if not args.no_cpu:
-        v, dt, threads, desc = cpu_sample(w, ratio, args.cpu_units, args.cpu_rows)
+        v, dt, threads, desc = cpu_sample(w, ratio, args.cpu_units, args.cpu_rows, args.path)
         line["cpu_baseline"] = {"value": v, "unit": "keys/s", "cores": threads,
                                 "kind": "oracle", "sample": desc, "seconds": dt}
     print(json.dumps(line), flush=True)
@@ -382,6 +402,9 @@ def main():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--e2e-chunk", type=int, default=0,
                     help="units per chunk of the host-buffer call (0: an eighth of L*H)")
+    ap.add_argument("--path", choices=("repair", "policy"), default="repair",
+                    help="repair: audit + swap (the headline); policy: the standalone "
+                         "scorer of Sec. 3.2")
     ap.add_argument("--layers", type=int, default=None,
                     help="fewer layers of the same workload (for profiler captures)")
     args = ap.parse_args()

@@ -108,14 +108,16 @@ typedef struct {
 typedef enum {
     TWINKV_OP_REDUNDANCY = 0,
     TWINKV_OP_REPAIR = 1,
-    TWINKV_OP_REPAIR_SELECT = 2
+    TWINKV_OP_REPAIR_SELECT = 2,
+    TWINKV_OP_POLICY = 3
 } twinkv_op;
 
 /* Kernels, for the profiling hooks. */
 typedef enum {
     TWINKV_KERNEL_PREP = 0,      /* bf16 rounding, norms, retained-first column gather */
     TWINKV_KERNEL_AUDIT = 1,     /* fused similarity + masked max/argmax (Eq. 1, Eq. 4) */
-    TWINKV_KERNEL_REPAIR = 2,    /* classify, rank, select and swap (Sec. 3.4) */
+    TWINKV_KERNEL_REPAIR = 2,    /* classify, rank, select and swap (Sec. 3.4); the
+                                    standalone policy's selection (Sec. 3.2, Eq. 3) */
     TWINKV_KERNEL_REFINE = 3,    /* exact value of each chosen twin's similarity (Eq. 1) */
     TWINKV_KERNEL_COUNT = 4
 } twinkv_kernel;
@@ -237,6 +239,34 @@ twinkv_status twinkv_repair_host(const void* keys, twinkv_shape s, const uint8_t
                                  int32_t* out_twin_all, int32_t* out_status,
                                  int32_t chunk_units, void* arena, size_t arena_bytes,
                                  void* stream);
+
+/*
+ * The standalone TwinKV policy (Sec. 3.2, Eq. 2-3): every key's redundancy count
+ *     r_i = #{ j : |i-j| > w, j != i, sim(i,j) > tau }          (Eq. 2, strict)
+ * and, per unit, the budget[u] positions with the highest score s_i = -r_i / N (Eq. 3),
+ * the sink and recent regions first (they carry the maximum score and tie among
+ * themselves), equal scores in position order (lower first).  All units in one pass;
+ * the N x N similarities are never stored.
+ *   keys        [L][H][N][d] device, dtype per s.dtype, 16-byte aligned
+ *   budget      [L*H] int32 device: positions kept per unit, e.g. ceil((1 - rho) N)
+ *               (Sec. 3.1); a budget below the protected count keeps the lowest
+ *               protected positions
+ *   threshold   tau (finite); overrides params->threshold
+ *   params      host pointer or NULL (defaults); window, n_sink, n_recent are used
+ *   out_mask    [L][H][N] uint8: 1 for a kept position
+ *   out_count   [L][H][N] int32: r_i, or NULL (then kept in the workspace)
+ *   out_status  [L*H] int32: 0, or TWINKV_ERR_INVALID_ARG where budget[u] is outside
+ *               [0, N] (that unit's mask is all 0); or NULL
+ * Precision: each pair is decided as the sign of one fp32 fused multiply-add,
+ * x_ij * (1/||k_j||) - tau * ||k_i||, x_ij the fp32 tensor-core dot product of the bf16
+ * keys: pairs whose similarity is within about 1e-6 of tau may count differently
+ * than in exact arithmetic.
+ * Workspace: twinkv_workspace_size(s, TWINKV_OP_POLICY) bytes, 256-byte aligned.
+ */
+twinkv_status twinkv_policy(const void* keys, twinkv_shape s, const int32_t* budget,
+                            float threshold, const twinkv_params* params, uint8_t* out_mask,
+                            int32_t* out_count, int32_t* out_status, void* workspace,
+                            size_t workspace_bytes, void* stream);
 
 /* Static description of a status code. */
 const char* twinkv_status_string(twinkv_status st);

@@ -20,7 +20,8 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libtwinkv.so")
-SOURCES = ["twk_api.cu", "twk_audit.cu", "twk_prep.cu", "twk_refine.cu", "twk_repair.cu"]
+SOURCES = ["twk_api.cu", "twk_audit.cu", "twk_prep.cu", "twk_refine.cu", "twk_repair.cu",
+           "twk_policy.cu"]
 HEADERS = ["twk_internal.h", "twk_ptx.cuh", "twk_df.cuh"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-I", INCLUDE, "-I", CSRC]

@@ -145,7 +145,7 @@ size_t up256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
 
 struct Layout {
     size_t keys16 = 0, colrinv = 0, colpos = 0, norm2 = 0, kp = 0, cnt = 0, kb = 0, twin0 = 0,
-           twin1 = 0, bret = 0, k0 = 0, i0 = 0, k1 = 0, i1 = 0;
+           twin1 = 0, bret = 0, k0 = 0, i0 = 0, k1 = 0, i1 = 0, rcount = 0;
     size_t total = 0;
 };
 
@@ -160,7 +160,7 @@ Layout layout(const twinkv_shape& s, int op)
     };
     const size_t U = static_cast<size_t>(s.L) * s.H;
     const size_t N = static_cast<size_t>(s.N);
-    if (op == TWINKV_OP_REDUNDANCY || op == TWINKV_OP_REPAIR) {
+    if (op == TWINKV_OP_REDUNDANCY || op == TWINKV_OP_REPAIR || op == TWINKV_OP_POLICY) {
         const size_t NP = static_cast<size_t>(column_stride(s.N));
         if (s.dtype == TWINKV_F32) L.keys16 = take(U * N * s.d * 2);
         L.colrinv = take(U * NP * 4);
@@ -175,6 +175,7 @@ Layout layout(const twinkv_shape& s, int op)
             L.bret = take(U * N * 8);
         }
     }
+    if (op == TWINKV_OP_POLICY) L.rcount = take(U * N * 4);
     if (op == TWINKV_OP_REPAIR || op == TWINKV_OP_REPAIR_SELECT) {
         L.k0 = take(U * N * 8);
         L.i0 = take(U * N * 4);
@@ -217,7 +218,8 @@ twinkv_status keys_bf16(const void* keys, const twinkv_shape& s, void* ws, const
 }
 
 twinkv_status run_audit(const DeviceInfo& dev, const twinkv_shape& s, const uint16_t* keys16,
-                        const void* bkeys, int64_t b_rows, AuditArgs a, cudaStream_t st)
+                        const void* bkeys, int64_t b_rows, AuditArgs a, cudaStream_t st,
+                        bool count = false)
 {
     CUtensorMap tmA, tmB;
     const int64_t U = static_cast<int64_t>(s.L) * s.H;
@@ -228,7 +230,7 @@ twinkv_status run_audit(const DeviceInfo& dev, const twinkv_shape& s, const uint
     const int64_t items = U * a.RB;
     const int grid = static_cast<int>(items < dev.sms ? items : dev.sms);
     ProfScope p(TWINKV_KERNEL_AUDIT, st);
-    return cuda_status(launch_audit(s.d, tmA, tmB, a, grid, st));
+    return cuda_status(launch_audit(s.d, count, tmA, tmB, a, grid, st));
 }
 
 twinkv_status params_ok(const twinkv_params& p, float threshold)
@@ -396,7 +398,7 @@ size_t twinkv_swaps_capacity(twinkv_shape s)
 
 size_t twinkv_workspace_size(twinkv_shape s, int32_t op)
 {
-    if (op < TWINKV_OP_REDUNDANCY || op > TWINKV_OP_REPAIR_SELECT) return 0;
+    if (op < TWINKV_OP_REDUNDANCY || op > TWINKV_OP_POLICY) return 0;
     if (!shape_ok(s, op != TWINKV_OP_REPAIR_SELECT)) return 0;
     return layout(s, op).total;
 }
@@ -545,6 +547,61 @@ twinkv_status twinkv_redundancy(const void* keys, twinkv_shape s, int32_t window
     if ((r = run_audit(*dev, s, k16, k16, static_cast<int64_t>(U) * s.N, a, st)) != TWINKV_OK)
         return r;
     return run_refine(k16, s, norm2, out_twin, nullptr, out_score, nullptr, st);
+}
+
+twinkv_status twinkv_policy(const void* keys, twinkv_shape s, const int32_t* budget,
+                            float threshold, const twinkv_params* params, uint8_t* out_mask,
+                            int32_t* out_count, int32_t* out_status, void* workspace,
+                            size_t workspace_bytes, void* stream)
+{
+    const twinkv_params p = params ? *params : twinkv_default_params();
+    if (!keys || !aligned16(keys) || !budget || !out_mask || !shape_ok(s, true))
+        return TWINKV_ERR_INVALID_ARG;
+    twinkv_status r = params_ok(p, threshold);
+    if (r != TWINKV_OK) return r;
+    Layout L;
+    if ((r = check_ws(s, TWINKV_OP_POLICY, workspace, workspace_bytes, &L)) != TWINKV_OK) return r;
+    DeviceInfo* dev = nullptr;
+    if ((r = device_info(&dev)) != TWINKV_OK) return r;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+
+    const uint16_t* k16 = nullptr;
+    if ((r = keys_bf16(keys, s, workspace, L, st, &k16)) != TWINKV_OK) return r;
+    const int U = s.L * s.H;
+    const int64_t NP = column_stride(s.N);
+    float* colrinv = at<float>(workspace, L.colrinv);
+    int* colpos = at<int>(workspace, L.colpos);
+    float4* norm2 = at<float4>(workspace, L.norm2);
+    int* count = out_count ? out_count : at<int>(workspace, L.rcount);
+    {
+        ProfScope pr(TWINKV_KERNEL_PREP, st);
+        if (launch_norms_identity(k16, U, s.N, s.d, NP, colrinv, colpos, norm2, st) !=
+            cudaSuccess)
+            return TWINKV_ERR_CUDA;
+    }
+    AuditArgs a;
+    std::memset(&a, 0, sizeof a);
+    a.U = U;
+    a.N = s.N;
+    a.NP = static_cast<int>(NP);
+    a.RB = (s.N + kBM - 1) / kBM;
+    a.window = p.window < s.N ? p.window : s.N;
+    a.repair_mode = 0;
+    a.need_all = 0;
+    a.b_rows_per_unit = s.N;
+    a.colrinv = colrinv;
+    a.colpos = colpos;
+    a.err = dev->err;
+    a.timeout_ns = g_timeout_ns;
+    a.mant_mask = 0xFFFFFFE0u;
+    a.count_tau = threshold;
+    a.out_count = count;
+    if ((r = run_audit(*dev, s, k16, k16, static_cast<int64_t>(U) * s.N, a, st, true)) !=
+        TWINKV_OK)
+        return r;
+    ProfScope pr(TWINKV_KERNEL_REPAIR, st);
+    return cuda_status(launch_policy_select(count, U, s.N, budget, p.n_sink, p.n_recent,
+                                            out_mask, out_status, st));
 }
 
 twinkv_status twinkv_repair(const void* keys, twinkv_shape s, const uint8_t* retained_mask,

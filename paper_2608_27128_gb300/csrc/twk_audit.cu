@@ -27,6 +27,12 @@
 // NaN): padding columns have 1/||k_j|| = NaN, and window columns (|i - j| <= w) are
 // set to NaN on the few tiles that intersect the window band of the row block.
 //
+// Count mode (Sec. 3.2 Eq. 2, the standalone scorer): instead of the maximum, each row i
+// counts the columns j outside the window with sim(i,j) > tau.  With x_ij the raw dot
+// product, that is x_ij * (1/||k_j||) > tau * ||k_i||, evaluated as the sign of one
+// fused multiply-add x_ij * (1/||k_j||) - tau / (1/||k_i||), so the product is never
+// rounded before the comparison; masked and padding columns are NaN and never count.
+//
 // Column layout: in repair mode the columns of a unit are stored retained-first
 // (retained keys in position order, padded to a tile, then evicted keys in position
 // order), so every tile belongs to exactly one of the two maxima.  The kernel writes
@@ -193,6 +199,54 @@ __device__ __forceinline__ void reduce_group(const uint32_t (&x0)[32], const uin
     fold32<kMasked>(x3, rinv + 96, pos + 96, rw, w2, mask, col0 + 96, b);
 }
 
+// 1 where a > b (false for NaN), as an all-ones word so that three-input integer adds
+// accumulate two comparisons per instruction.
+__device__ __forceinline__ uint32_t gt_mask(float a, float b)
+{
+    uint32_t r;
+    asm("set.gt.u32.f32 %0, %1, %2;" : "=r"(r) : "f"(a), "f"(b));
+    return r;
+}
+
+// Eq. 2 over 32 columns: how many x_j / ||k_j|| exceed t = tau * ||k_i||.
+template <bool kMasked>
+__device__ __forceinline__ int count32(const uint32_t (&x)[32], const float* rinv,
+                                       const int* pos, int rw, uint32_t w2, float t)
+{
+    int c = 0;
+    const float2 mt = make_float2(-t, -t);
+#pragma unroll
+    for (int k = 0; k < 32; k += 4) {
+        const float4 r = *reinterpret_cast<const float4*>(rinv + k);
+        float2 a = make_float2(__uint_as_float(x[k]), __uint_as_float(x[k + 1]));
+        float2 b = make_float2(__uint_as_float(x[k + 2]), __uint_as_float(x[k + 3]));
+        if (kMasked) {
+            const int4 q = *reinterpret_cast<const int4*>(pos + k);
+            a.x = (static_cast<uint32_t>(q.x - rw) > w2) ? a.x : nan_f();
+            a.y = (static_cast<uint32_t>(q.y - rw) > w2) ? a.y : nan_f();
+            b.x = (static_cast<uint32_t>(q.z - rw) > w2) ? b.x : nan_f();
+            b.y = (static_cast<uint32_t>(q.w - rw) > w2) ? b.y : nan_f();
+        }
+        const float2 fa = __ffma2_rn(a, make_float2(r.x, r.y), mt);
+        const float2 fb = __ffma2_rn(b, make_float2(r.z, r.w), mt);
+        c -= static_cast<int>(gt_mask(fa.x, 0.f)) + static_cast<int>(gt_mask(fa.y, 0.f));
+        c -= static_cast<int>(gt_mask(fb.x, 0.f)) + static_cast<int>(gt_mask(fb.y, 0.f));
+    }
+    return c;
+}
+
+template <bool kMasked>
+__device__ __forceinline__ int count_group(const uint32_t (&x0)[32], const uint32_t (&x1)[32],
+                                           const uint32_t (&x2)[32], const uint32_t (&x3)[32],
+                                           const float* rinv, const int* pos, int rw,
+                                           uint32_t w2, float t)
+{
+    return count32<kMasked>(x0, rinv, pos, rw, w2, t) +
+           count32<kMasked>(x1, rinv + 32, pos + 32, rw, w2, t) +
+           count32<kMasked>(x2, rinv + 64, pos + 64, rw, w2, t) +
+           count32<kMasked>(x3, rinv + 96, pos + 96, rw, w2, t);
+}
+
 struct Tiles {
     int tr;   // tiles of segment 0 (retained, or every column in mode 0)
     int te;   // tiles of segment 1 (evicted; 0 unless b_all is wanted)
@@ -242,7 +296,7 @@ __device__ __forceinline__ int last_parity(long long total, int n, int s)
 
 // Registers are per sub-partition (16384 each): with W warps a sub-partition holds
 // ceil(W / 4) of them, which bounds the registers per thread.
-template <int D>
+template <int D, bool kCount>
 __global__ void __launch_bounds__(kThreads, 1)
     audit_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                  const __grid_constant__ AuditArgs a)
@@ -477,6 +531,9 @@ __global__ void __launch_bounds__(kThreads, 1)
 
             Best b0{-INFINITY, -1}, b1{-INFINITY, -1};   // retained (or all) / evicted
             const int rw = row - w;
+            int cnt = 0;                                   // count mode: r_i so far
+            float thr = 0.f;                               // count mode: tau * ||k_i||
+            if (kCount) thr = a.count_tau / a.colrinv[static_cast<int64_t>(u) * a.NP + row];
             for (int t = 0; t < nt; ++t) {
                 ok = all_wait(&m_full[ms], mph, wc, 7);
                 if (ok) ok = all_wait(&t_full[acc], tph, wc, 8);
@@ -496,7 +553,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                 tc_fence_before();
                 __syncwarp();
                 if (lane == 0) mbar_arrive(&t_empty[acc]);
-                if (t < ut.tr) {
+                if (kCount) {
+                    cnt += band ? count_group<true>(x0, x1, x2, x3, rinv, pos, rw, w2, thr)
+                                : count_group<false>(x0, x1, x2, x3, rinv, pos, rw, w2, thr);
+                } else if (t < ut.tr) {
                     if (band) reduce_group<true>(x0, x1, x2, x3, rinv, pos, rw, w2, mask, c_lo, b0);
                     else reduce_group<false>(x0, x1, x2, x3, rinv, pos, rw, w2, mask, c_lo, b0);
                 } else {
@@ -531,8 +591,18 @@ __global__ void __launch_bounds__(kThreads, 1)
                 ok = all_wait(&x_empty[xb], ((n_x >> 1) & 1) ^ 1, wc, 9);
                 if (!ok) break;
                 X[(h - 1) * kBM + row_local] =
-                    make_float4(bv0, __int_as_float(bc0), bv1, __int_as_float(bc1));
+                    kCount ? make_float4(__int_as_float(cnt), 0.f, 0.f, 0.f)
+                           : make_float4(bv0, __int_as_float(bc0), bv1, __int_as_float(bc1));
                 mbar_arrive(&x_full[xb]);
+            } else if (kCount) {
+                ok = all_wait(&x_full[xb], (n_x >> 1) & 1, wc, 10);
+                if (!ok) break;
+                int total = cnt;
+#pragma unroll
+                for (int g = 1; g < kGroups; ++g)
+                    total += __float_as_int(X[(g - 1) * kBM + row_local].x);
+                mbar_arrive(&x_empty[xb]);
+                if (row < a.N) a.out_count[static_cast<int64_t>(u) * a.N + row] = total;
             } else {
                 ok = all_wait(&x_full[xb], (n_x >> 1) & 1, wc, 10);
                 if (!ok) break;
@@ -578,23 +648,26 @@ size_t audit_smem_bytes(int d)
     return d == 128 ? AuditCfg<128>::BYTES : AuditCfg<64>::BYTES;
 }
 
-cudaError_t launch_audit(int d, const CUtensorMap& tmA, const CUtensorMap& tmB,
+template <int D, bool kCount>
+cudaError_t launch_audit_t(const CUtensorMap& tmA, const CUtensorMap& tmB, const AuditArgs& a,
+                           int grid, cudaStream_t st)
+{
+    const int bytes = AuditCfg<D>::BYTES;
+    cudaError_t e = cudaFuncSetAttribute(audit_kernel<D, kCount>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+    if (e != cudaSuccess) return e;
+    audit_kernel<D, kCount><<<grid, kThreads, bytes, st>>>(tmA, tmB, a);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_audit(int d, bool count, const CUtensorMap& tmA, const CUtensorMap& tmB,
                          const AuditArgs& a, int grid, cudaStream_t st)
 {
-    if (d == 128) {
-        const int bytes = AuditCfg<128>::BYTES;
-        cudaError_t e = cudaFuncSetAttribute(audit_kernel<128>,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
-        if (e != cudaSuccess) return e;
-        audit_kernel<128><<<grid, kThreads, bytes, st>>>(tmA, tmB, a);
-    } else {
-        const int bytes = AuditCfg<64>::BYTES;
-        cudaError_t e = cudaFuncSetAttribute(audit_kernel<64>,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
-        if (e != cudaSuccess) return e;
-        audit_kernel<64><<<grid, kThreads, bytes, st>>>(tmA, tmB, a);
-    }
-    return cudaGetLastError();
+    if (d == 128)
+        return count ? launch_audit_t<128, true>(tmA, tmB, a, grid, st)
+                     : launch_audit_t<128, false>(tmA, tmB, a, grid, st);
+    return count ? launch_audit_t<64, true>(tmA, tmB, a, grid, st)
+                 : launch_audit_t<64, false>(tmA, tmB, a, grid, st);
 }
 
 // ---------------------------------------------------------------- wait probe

@@ -33,6 +33,9 @@ struct AuditArgs {
     uint32_t mant_mask;         // 0xFFFFFFE0: clears the 5 mantissa bits that carry the
                                 // column; a runtime value, so the compiler keeps it in a
                                 // register and the pack is a single 3-input logic op
+    // count mode (Eq. 2): mode 0 columns only; out_t0/out_t1 unused
+    float count_tau;            // tau, compared strictly
+    int* out_count;             // [U][N] r_i
 };
 
 struct RepairArgs {
@@ -73,8 +76,15 @@ cudaError_t launch_refine(const uint16_t* keys, int U, int N, int d, const float
 
 // audit kernel (tensor maps built by the caller)
 size_t audit_smem_bytes(int d);
-cudaError_t launch_audit(int d, const CUtensorMap& tmA, const CUtensorMap& tmB,
+// count = false: max/argmax (Eq. 1, Eq. 4); true: redundancy counts (Eq. 2)
+cudaError_t launch_audit(int d, bool count, const CUtensorMap& tmA, const CUtensorMap& tmB,
                          const AuditArgs& a, int grid, cudaStream_t st);
+
+// standalone policy selection (Sec. 3.2, Eq. 3): per unit, keep budget[u] positions
+// ordered by (protected first, count ascending, position ascending)
+cudaError_t launch_policy_select(const int* count, int U, int N, const int* budget, int n_sink,
+                                 int n_recent, uint8_t* out_mask, int* out_status,
+                                 cudaStream_t st);
 
 // repair kernel
 cudaError_t launch_repair(const RepairArgs& a, cudaStream_t st);

@@ -11,6 +11,7 @@ Sec. 3.4 (Eq. 4, orphans, donors, the budget-exact swap).
 from __future__ import annotations
 
 import ctypes
+import math
 import os
 import threading
 
@@ -22,7 +23,7 @@ from . import build as _build
  ERR_TOO_LARGE) = range(8)
 NOALLOC_MAX_POSITIONS = 262144
 BF16, F32 = 0, 1
-OP_REDUNDANCY, OP_REPAIR, OP_REPAIR_SELECT = 0, 1, 2
+OP_REDUNDANCY, OP_REPAIR, OP_REPAIR_SELECT, OP_POLICY = 0, 1, 2, 3
 KERNEL_PREP, KERNEL_AUDIT, KERNEL_REPAIR, KERNEL_REFINE = 0, 1, 2, 3
 KERNEL_NAMES = ("prep", "audit", "repair", "refine")
 
@@ -32,6 +33,7 @@ EXPORTED = (
     "twinkv_status_string", "twinkv_get_last_error", "twinkv_set_wait_timeout_ns",
     "twinkv_wait_probe", "twinkv_profile_begin", "twinkv_profile_end",
     "twinkv_repair_select_noalloc", "twinkv_host_arena_size", "twinkv_repair_host",
+    "twinkv_policy",
 )
 
 
@@ -95,6 +97,8 @@ def load(build_if_missing: bool = True):
         lib.twinkv_repair_host.argtypes = [_P, Shape, _P, _P, ctypes.c_float,
                                            ctypes.POINTER(Params), _P, _P, _P, _P, _P, _P, _P,
                                            _P, ctypes.c_int32, _P, ctypes.c_size_t, _P]
+        lib.twinkv_policy.argtypes = [_P, Shape, _P, ctypes.c_float, ctypes.POINTER(Params),
+                                      _P, _P, _P, _P, ctypes.c_size_t, _P]
         lib.twinkv_status_string.argtypes = [ctypes.c_int]
         lib.twinkv_status_string.restype = ctypes.c_char_p
         lib.twinkv_set_wait_timeout_ns.argtypes = [ctypes.c_uint64]
@@ -102,7 +106,7 @@ def load(build_if_missing: bool = True):
         lib.twinkv_profile_end.argtypes = [ctypes.POINTER(ctypes.c_int32),
                                            ctypes.POINTER(ctypes.c_double)]
         for name in ("twinkv_redundancy", "twinkv_repair", "twinkv_repair_select",
-                     "twinkv_repair_select_noalloc", "twinkv_repair_host",
+                     "twinkv_repair_select_noalloc", "twinkv_repair_host", "twinkv_policy",
                      "twinkv_get_last_error", "twinkv_set_wait_timeout_ns",
                      "twinkv_wait_probe", "twinkv_profile_begin", "twinkv_profile_end"):
             getattr(lib, name).restype = ctypes.c_int
@@ -326,6 +330,43 @@ def twinkv_repair_select_noalloc(score_ret, retained_mask, budget=None, threshol
         ctypes.byref(p), _ptr(o["mask"]), _ptr(o["swaps"]), _ptr(o["nswaps"]),
         _ptr(o["status"]), _stream(stream))
     _check(st, "twinkv_repair_select_noalloc")
+    return o
+
+
+def budget_for_ratio(N: int, ratio: float) -> int:
+    """Retained count of Sec. 3.1: |S| = ceil((1 - rho) n)."""
+    return int(math.ceil((1.0 - float(ratio)) * N - 1e-9))
+
+
+def twinkv_policy(keys, budget, threshold=None, params=None, *, window=None, n_sink=None,
+                  n_recent=None, want_count=True, out=None, ws=None, stream=None) -> dict:
+    """The standalone TwinKV policy (Sec. 3.2, Eq. 2-3) on keys [L,H,N,d].
+
+    budget: int32 CUDA tensor [L*H], or an int used for every unit.  Returns a dict of
+    CUDA tensors: mask [L,H,N] uint8 (kept positions), status [L*H] int32 and, with
+    want_count, count [L,H,N] int32 (r_i of Eq. 2).
+    """
+    s = shape_of(keys)
+    dev = keys.device
+    _need(keys, "keys", keys.dtype, keys.shape, dev)
+    L, H, N = s.L, s.H, s.N
+    if not isinstance(budget, torch.Tensor):
+        budget = torch.full((L * H,), int(budget), dtype=torch.int32, device=dev)
+    _need(budget, "budget", torch.int32, (L * H,), dev)
+    p = _params(params, threshold, window, n_sink, n_recent)
+    out = dict(out or {})
+    o = {
+        "mask": _out(out.get("mask"), "mask", torch.uint8, (L, H, N), dev),
+        "status": _out(out.get("status"), "status", torch.int32, (L * H,), dev),
+    }
+    if want_count:
+        o["count"] = _out(out.get("count"), "count", torch.int32, (L, H, N), dev)
+    ws = _ws(ws, s, OP_POLICY, dev)
+    st = load().twinkv_policy(
+        _ptr(keys), s, _ptr(budget), ctypes.c_float(p.threshold), ctypes.byref(p),
+        _ptr(o["mask"]), _ptr(o.get("count")), _ptr(o["status"]), _ptr(ws), ws.numel(),
+        _stream(stream))
+    _check(st, "twinkv_policy")
     return o
 
 
