@@ -13,6 +13,7 @@ from .oracle import (  # noqa: F401
     policy,
     policy_select,
     repair,
+    repair_dedup,
     repair_f32,
     round_bf16,
     sim,

@@ -56,6 +56,9 @@ def _load():
                 ctypes.c_double, _P, ctypes.c_int, _P, _P, _P]
             lib.twk_oracle_policy_select.argtypes = [
                 ctypes.c_int, ctypes.c_int, _P, ctypes.c_int, ctypes.c_int, _P, _P, _P]
+            lib.twk_oracle_repair_dedup.argtypes = [
+                ctypes.c_int, ctypes.c_int, _P, _P, _P, _P, ctypes.c_float, ctypes.c_int,
+                ctypes.c_int, _P, _P, _P, _P]
             for name in ("twk_oracle_repair", "twk_oracle_repair_f32"):
                 getattr(lib, name).argtypes = [
                     ctypes.c_int, ctypes.c_int, _P, _P, _P, ctypes.c_float, ctypes.c_int,
@@ -205,3 +208,31 @@ def policy(keys, threshold: float, budget, window: int = 32, n_sink: int = 4,
     c = count(keys, threshold, window)
     p = policy_select(c["r"], budget, n_sink, n_recent)
     return {"r": c["r"], **p}
+
+
+def repair_dedup(b_ret, t_ret, mask, threshold: float, n_sink: int = 4, n_recent: int = 64,
+                 budget=None) -> dict:
+    """Sec. 3.4 repair that never evicts both members of a twin pair: donors walked in
+    severity order, a donor skipped when its twin (t_ret) is already being evicted or
+    when it is the twin of an evicted donor.
+    b_ret fp64 [U,N], t_ret int32 [U,N]."""
+    b = np.ascontiguousarray(np.asarray(b_ret, dtype=np.float64))
+    U = b.shape[0] if b.ndim == 2 else 1
+    b = b.reshape(U, -1)
+    N = b.shape[1]
+    t = np.ascontiguousarray(np.asarray(t_ret, dtype=np.int32).reshape(U, N))
+    m = np.ascontiguousarray(np.asarray(mask, dtype=np.uint8).reshape(U, N))
+    bud = None
+    if budget is not None:
+        bud = np.ascontiguousarray(np.asarray(budget, dtype=np.int32).reshape(U))
+    out = {
+        "mask": np.empty((U, N), np.uint8),
+        "swaps": np.full((U, N // 2, 2), -1, np.int32),
+        "nswaps": np.empty(U, np.int32),
+        "status": np.empty(U, np.int32),
+    }
+    _load().twk_oracle_repair_dedup(U, N, _ptr(b), _ptr(t), _ptr(m), _ptr(bud),
+                                    ctypes.c_float(threshold), int(n_sink), int(n_recent),
+                                    _ptr(out["mask"]), _ptr(out["swaps"]), _ptr(out["nswaps"]),
+                                    _ptr(out["status"]))
+    return out

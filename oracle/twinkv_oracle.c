@@ -25,6 +25,9 @@
  *   Sec. 3.4, repair     rank orphans by ascending b, donors by descending b,
  *                        m = min(|O|,|D|), evict the m most severe donors and admit
  *                        the m most severe orphans; |S1| = |S0|
+ *   (dedup variant)      the repair with donors taken in severity order, where evicting
+ *                        a donor keeps its twin (its b_i(S0) argmax) in place, so a
+ *                        twin pair never loses both members
  *   Sec. 3.2, Eq. 2      r_i = number of j with |i-j| > w (j != i) and sim(i,j) > tau
  *   Sec. 3.2, Eq. 3      s_i = -r_i / n; the standalone policy keeps the K highest
  *                        scores, with the sink and recent regions given the maximum
@@ -40,6 +43,11 @@
  *     so that a float implementation and this oracle compare against the same number;
  *   - keys are bf16 bit patterns; float32 keys are first rounded to bf16,
  *     round-to-nearest-even;
+ *   - the dedup variant is this build's reading of the paper's remark that one member
+ *     of a twin pair already holds a slot (Sec. 3.4): walking donors from the most
+ *     severe, a donor is skipped when its twin was accepted for eviction earlier in
+ *     the walk, or when it is the twin of an accepted donor (it now holds that
+ *     donor's content); the walk stops after |O| accepted donors;
  *   - the standalone policy orders positions by (protected first, r ascending, i.e.
  *     s descending, then position ascending) and keeps the first K; a budget below
  *     the protected count keeps the lowest protected positions.
@@ -410,4 +418,93 @@ void twk_oracle_policy_select(int U, int N, const int32_t* r, int n_sink, int n_
             S[e[k].pos] = 1;
     }
     free(e);
+}
+
+/* ---- Sec. 3.4 variant: the repair without evicting both members of a twin pair -- */
+
+/*
+ * Like twk_oracle_repair, with twin[U][N] = the argmax of b_i(S0) (Eq. 4) per
+ * position.  Donors are walked in severity order (b descending, position ascending);
+ * a donor is skipped when its twin has already been accepted for eviction in this
+ * walk, or when it is itself the twin of an accepted donor; the walk stops once |O|
+ * donors are accepted.  m = the number accepted; the m
+ * most severe orphans are admitted, the k-th accepted donor paired with the k-th
+ * orphan.  Status handling as in twk_oracle_repair.
+ */
+void twk_oracle_repair_dedup(int U, int N, const double* b, const int32_t* twin,
+                             const uint8_t* mask, const int32_t* budget, float threshold,
+                             int n_sink, int n_recent, uint8_t* out_mask, int32_t* swaps,
+                             int32_t* nswaps, int32_t* status)
+{
+    const double tau = (double)threshold;
+    const long cap = 2L * (N / 2);
+    ranked* orphans = (ranked*)malloc(sizeof(ranked) * (size_t)(N > 0 ? N : 1));
+    ranked* donors = (ranked*)malloc(sizeof(ranked) * (size_t)(N > 0 ? N : 1));
+    uint8_t* evicted = (uint8_t*)malloc((size_t)(N > 0 ? N : 1));
+    uint8_t* pinned = (uint8_t*)malloc((size_t)(N > 0 ? N : 1));
+    for (int u = 0; u < U; ++u) {
+        const uint8_t* S0 = mask + (long)u * N;
+        const double* bu = b + (long)u * N;
+        const int32_t* tw = twin + (long)u * N;
+        uint8_t* S1 = out_mask + (long)u * N;
+        int32_t* sw = swaps + (long)u * cap;
+        int bad_value = 0, count = 0;
+        for (int i = 0; i < N; ++i) {
+            if (S0[i] > 1) bad_value = 1;
+            count += S0[i] != 0;
+        }
+        int st = 0;
+        if (bad_value)
+            st = 1;
+        else if (budget && budget[u] != count)
+            st = 3;
+        status[u] = st;
+        memcpy(S1, S0, (size_t)N);
+        if (st != 0) {
+            nswaps[u] = -1;
+            continue;
+        }
+        int n_o = 0, n_d = 0;
+        for (int i = 0; i < N; ++i) {
+            int retained = S0[i] != 0;
+            int protected_pos = (i < n_sink) || (i >= N - n_recent);
+            if (!retained && bu[i] < tau) {
+                orphans[n_o].b = bu[i];
+                orphans[n_o].pos = i;
+                ++n_o;
+            }
+            if (retained && !protected_pos && bu[i] >= tau) {
+                donors[n_d].b = bu[i];
+                donors[n_d].pos = i;
+                ++n_d;
+            }
+        }
+        qsort(orphans, (size_t)n_o, sizeof(ranked), cmp_orphan);
+        qsort(donors, (size_t)n_d, sizeof(ranked), cmp_donor);
+        memset(evicted, 0, (size_t)N);
+        memset(pinned, 0, (size_t)N);
+        int m = 0;
+        for (int k = 0; k < n_d && m < n_o; ++k) {
+            int d = donors[k].pos;
+            int t = tw[d];
+            int has_twin = t >= 0 && t < N;
+            if (pinned[d] || (has_twin && evicted[t]))
+                continue;
+            evicted[d] = 1;
+            if (has_twin)
+                pinned[t] = 1;
+            sw[2 * m] = d;
+            ++m;
+        }
+        for (int k = 0; k < m; ++k) {
+            sw[2 * k + 1] = orphans[k].pos;
+            S1[sw[2 * k]] = 0;
+            S1[orphans[k].pos] = 1;
+        }
+        nswaps[u] = m;
+    }
+    free(orphans);
+    free(donors);
+    free(evicted);
+    free(pinned);
 }
