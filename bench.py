@@ -46,8 +46,9 @@ def peaks():
 
 
 def workload_config(w, ratio, path="repair"):
-    what = ("audit + repair (Sec. 3.4)" if path == "repair"
-            else "standalone policy: counts + selection (Sec. 3.2 Eq. 2-3)")
+    what = {"repair": "audit + repair (Sec. 3.4)",
+            "dedup": "audit + repair that keeps one member of each twin pair (Sec. 3.4)",
+            "policy": "standalone policy: counts + selection (Sec. 3.2 Eq. 2-3)"}[path]
     return {
         "workload": f"Qwen3-4B KV cache {w.L}x{w.H}x{w.N}x{w.d} bf16 (synthetic), ratio {ratio}, "
                     f"{what}",
@@ -235,6 +236,8 @@ def run_ours(args, w, ratio):
         nonlocal out
         if args.path == "policy":
             out = tk.twinkv_policy(k, K, threshold=w.tau, out=out, ws=ws)
+        elif args.path == "dedup":
+            out = tk.twinkv_repair_dedup(k, m, b, threshold=w.tau, want_all=True, out=out, ws=ws)
         else:
             out = tk.twinkv_repair(k, m, b, threshold=w.tau, want_all=True, out=out, ws=ws)
         return out
@@ -328,7 +331,7 @@ def _report(args, w, ratio, world, U, N, d, ms, prof, e2e_ms, h2d, d2h, chunk, c
     achieved = flops / (audit_ms_per * 1e-3) / 1e12
     peak = pk["bf16_tflops_sustained"]
     launches = sum(n for n, _ in prof.values())
-    traffic = audit_traffic(U) if args.path == "repair" else None
+    traffic = audit_traffic(U) if args.path in ("repair", "dedup") else None
 
     line = {
         "metric": METRIC, "value": value, "unit": "keys/s", "n_gpus": world,
@@ -402,9 +405,10 @@ def main():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--e2e-chunk", type=int, default=0,
                     help="units per chunk of the host-buffer call (0: an eighth of L*H)")
-    ap.add_argument("--path", choices=("repair", "policy"), default="repair",
-                    help="repair: audit + swap (the headline); policy: the standalone "
-                         "scorer of Sec. 3.2")
+    ap.add_argument("--path", choices=("repair", "dedup", "policy"), default="repair",
+                    help="repair: audit + swap (the headline); dedup: the repair that "
+                         "never evicts both members of a twin pair; policy: the "
+                         "standalone scorer of Sec. 3.2")
     ap.add_argument("--layers", type=int, default=None,
                     help="fewer layers of the same workload (for profiler captures)")
     args = ap.parse_args()

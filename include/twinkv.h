@@ -109,7 +109,8 @@ typedef enum {
     TWINKV_OP_REDUNDANCY = 0,
     TWINKV_OP_REPAIR = 1,
     TWINKV_OP_REPAIR_SELECT = 2,
-    TWINKV_OP_POLICY = 3
+    TWINKV_OP_POLICY = 3,
+    TWINKV_OP_REPAIR_SELECT_DEDUP = 4
 } twinkv_op;
 
 /* Kernels, for the profiling hooks. */
@@ -239,6 +240,41 @@ twinkv_status twinkv_repair_host(const void* keys, twinkv_shape s, const uint8_t
                                  int32_t* out_twin_all, int32_t* out_status,
                                  int32_t chunk_units, void* arena, size_t arena_bytes,
                                  void* stream);
+
+/*
+ * twinkv_repair with a donor never evicted together with its twin (Sec. 3.4: a donor
+ * is redundant because its twin, the argmax of b_i(S0), holds the same content; the
+ * literal rule can still evict both members of a retained twin pair).  Donors are
+ * walked in severity order (b descending, position ascending); a donor is skipped when
+ * its twin is already being evicted, or when it is the twin of an evicted donor; the
+ * walk stops after |O| evictions, so m = the number of evictions <= min(|O|, |D|).  The
+ * m most severe orphans are admitted, the k-th evicted donor paired with the k-th
+ * orphan.  Arguments, outputs and the workspace (TWINKV_OP_REPAIR) as for
+ * twinkv_repair; N must not exceed 524288 (TWINKV_ERR_UNSUPPORTED otherwise: the walk
+ * keeps two bits per donor in shared memory).  The walk is sequential per unit, so a
+ * unit with many donors takes longer than in twinkv_repair.
+ */
+twinkv_status twinkv_repair_dedup(const void* keys, twinkv_shape s, const uint8_t* retained_mask,
+                                  const int32_t* budget, float threshold,
+                                  const twinkv_params* params, uint8_t* out_mask,
+                                  int32_t* out_swaps, int32_t* out_nswaps, double* out_score_ret,
+                                  int32_t* out_twin_ret, double* out_score_all,
+                                  int32_t* out_twin_all, int32_t* out_status, void* workspace,
+                                  size_t workspace_bytes, void* stream);
+
+/*
+ * The selection of twinkv_repair_dedup alone, on caller-supplied b_i(S0) and twins.
+ *   score_ret   [L][H][N] float64 device, b_i(S0)
+ *   twin_ret    [L][H][N] int32 device, the position of each b_i(S0)'s argmax (-1 none)
+ *   other arguments as for twinkv_repair_select; workspace TWINKV_OP_REPAIR_SELECT_DEDUP
+ */
+twinkv_status twinkv_repair_select_dedup(const double* score_ret, const int32_t* twin_ret,
+                                         twinkv_shape s, const uint8_t* retained_mask,
+                                         const int32_t* budget, float threshold,
+                                         const twinkv_params* params, uint8_t* out_mask,
+                                         int32_t* out_swaps, int32_t* out_nswaps,
+                                         int32_t* out_status, void* workspace,
+                                         size_t workspace_bytes, void* stream);
 
 /*
  * The standalone TwinKV policy (Sec. 3.2, Eq. 2-3): every key's redundancy count

@@ -145,7 +145,7 @@ size_t up256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
 
 struct Layout {
     size_t keys16 = 0, colrinv = 0, colpos = 0, norm2 = 0, kp = 0, cnt = 0, kb = 0, twin0 = 0,
-           twin1 = 0, bret = 0, k0 = 0, i0 = 0, k1 = 0, i1 = 0, rcount = 0;
+           twin1 = 0, bret = 0, k0 = 0, i0 = 0, k1 = 0, i1 = 0, rcount = 0, rank = 0;
     size_t total = 0;
 };
 
@@ -176,11 +176,13 @@ Layout layout(const twinkv_shape& s, int op)
         }
     }
     if (op == TWINKV_OP_POLICY) L.rcount = take(U * N * 4);
-    if (op == TWINKV_OP_REPAIR || op == TWINKV_OP_REPAIR_SELECT) {
+    if (op == TWINKV_OP_REPAIR || op == TWINKV_OP_REPAIR_SELECT ||
+        op == TWINKV_OP_REPAIR_SELECT_DEDUP) {
         L.k0 = take(U * N * 8);
         L.i0 = take(U * N * 4);
         L.k1 = take(U * N * 8);
         L.i1 = take(U * N * 4);
+        if (op != TWINKV_OP_REPAIR_SELECT) L.rank = take(U * N * 4);   // dedup's rank table
     }
     L.total = off;
     return L;
@@ -243,7 +245,8 @@ twinkv_status params_ok(const twinkv_params& p, float threshold)
 twinkv_status launch_select(const twinkv_shape& s, const double* b, const uint8_t* mask,
                             const int32_t* budget, float threshold, const twinkv_params& p,
                             uint8_t* out_mask, int32_t* out_swaps, int32_t* out_nswaps,
-                            int32_t* out_status, void* ws, const Layout& L, cudaStream_t st)
+                            int32_t* out_status, void* ws, const Layout& L, cudaStream_t st,
+                            const int32_t* twin = nullptr)
 {
     RepairArgs r;
     r.U = s.L * s.H;
@@ -262,6 +265,9 @@ twinkv_status launch_select(const twinkv_shape& s, const double* b, const uint8_
     r.idx0 = at<int>(ws, L.i0);
     r.keys1 = at<uint64_t>(ws, L.k1);
     r.idx1 = at<int>(ws, L.i1);
+    r.twin = twin;
+    r.rank_of = twin ? at<int>(ws, L.rank) : nullptr;
+    if (twin && s.N > kDedupMaxN) return TWINKV_ERR_UNSUPPORTED;
     ProfScope prof(TWINKV_KERNEL_REPAIR, st);
     return cuda_status(launch_repair(r, st));
 }
@@ -398,8 +404,9 @@ size_t twinkv_swaps_capacity(twinkv_shape s)
 
 size_t twinkv_workspace_size(twinkv_shape s, int32_t op)
 {
-    if (op < TWINKV_OP_REDUNDANCY || op > TWINKV_OP_POLICY) return 0;
-    if (!shape_ok(s, op != TWINKV_OP_REPAIR_SELECT)) return 0;
+    if (op < TWINKV_OP_REDUNDANCY || op > TWINKV_OP_REPAIR_SELECT_DEDUP) return 0;
+    if (!shape_ok(s, op != TWINKV_OP_REPAIR_SELECT && op != TWINKV_OP_REPAIR_SELECT_DEDUP))
+        return 0;
     return layout(s, op).total;
 }
 
@@ -604,12 +611,15 @@ twinkv_status twinkv_policy(const void* keys, twinkv_shape s, const int32_t* bud
                                             out_mask, out_status, st));
 }
 
-twinkv_status twinkv_repair(const void* keys, twinkv_shape s, const uint8_t* retained_mask,
-                            const int32_t* budget, float threshold, const twinkv_params* params,
-                            uint8_t* out_mask, int32_t* out_swaps, int32_t* out_nswaps,
-                            double* out_score_ret, int32_t* out_twin_ret, double* out_score_all,
-                            int32_t* out_twin_all, int32_t* out_status, void* workspace,
-                            size_t workspace_bytes, void* stream)
+}  // extern "C"
+
+namespace {
+twinkv_status repair_impl(const void* keys, twinkv_shape s, const uint8_t* retained_mask,
+                          const int32_t* budget, float threshold, const twinkv_params* params,
+                          uint8_t* out_mask, int32_t* out_swaps, int32_t* out_nswaps,
+                          double* out_score_ret, int32_t* out_twin_ret, double* out_score_all,
+                          int32_t* out_twin_all, int32_t* out_status, void* workspace,
+                          size_t workspace_bytes, void* stream, bool dedup)
 {
     const twinkv_params p = params ? *params : twinkv_default_params();
     if (!keys || !aligned16(keys) || !retained_mask || !out_mask || !out_nswaps ||
@@ -671,7 +681,60 @@ twinkv_status twinkv_repair(const void* keys, twinkv_shape s, const uint8_t* ret
     if ((r = run_refine(k16, s, norm2, t0, t1, bret, out_score_all, st)) != TWINKV_OK)
         return r;
     return launch_select(s, bret, retained_mask, budget, threshold, p, out_mask, out_swaps,
-                         out_nswaps, out_status, workspace, L, st);
+                         out_nswaps, out_status, workspace, L, st, dedup ? t0 : nullptr);
+}
+}  // namespace
+
+extern "C" {
+
+twinkv_status twinkv_repair(const void* keys, twinkv_shape s, const uint8_t* retained_mask,
+                            const int32_t* budget, float threshold, const twinkv_params* params,
+                            uint8_t* out_mask, int32_t* out_swaps, int32_t* out_nswaps,
+                            double* out_score_ret, int32_t* out_twin_ret, double* out_score_all,
+                            int32_t* out_twin_all, int32_t* out_status, void* workspace,
+                            size_t workspace_bytes, void* stream)
+{
+    return repair_impl(keys, s, retained_mask, budget, threshold, params, out_mask, out_swaps,
+                       out_nswaps, out_score_ret, out_twin_ret, out_score_all, out_twin_all,
+                       out_status, workspace, workspace_bytes, stream, false);
+}
+
+twinkv_status twinkv_repair_dedup(const void* keys, twinkv_shape s, const uint8_t* retained_mask,
+                                  const int32_t* budget, float threshold,
+                                  const twinkv_params* params, uint8_t* out_mask,
+                                  int32_t* out_swaps, int32_t* out_nswaps, double* out_score_ret,
+                                  int32_t* out_twin_ret, double* out_score_all,
+                                  int32_t* out_twin_all, int32_t* out_status, void* workspace,
+                                  size_t workspace_bytes, void* stream)
+{
+    return repair_impl(keys, s, retained_mask, budget, threshold, params, out_mask, out_swaps,
+                       out_nswaps, out_score_ret, out_twin_ret, out_score_all, out_twin_all,
+                       out_status, workspace, workspace_bytes, stream, true);
+}
+
+twinkv_status twinkv_repair_select_dedup(const double* score_ret, const int32_t* twin_ret,
+                                         twinkv_shape s, const uint8_t* retained_mask,
+                                         const int32_t* budget, float threshold,
+                                         const twinkv_params* params, uint8_t* out_mask,
+                                         int32_t* out_swaps, int32_t* out_nswaps,
+                                         int32_t* out_status, void* workspace,
+                                         size_t workspace_bytes, void* stream)
+{
+    const twinkv_params p = params ? *params : twinkv_default_params();
+    if (!score_ret || !twin_ret || !retained_mask || !out_mask || !out_nswaps ||
+        !shape_ok(s, false) || (!out_swaps && s.N >= 2))
+        return TWINKV_ERR_INVALID_ARG;
+    twinkv_status r = params_ok(p, threshold);
+    if (r != TWINKV_OK) return r;
+    Layout L;
+    if ((r = check_ws(s, TWINKV_OP_REPAIR_SELECT_DEDUP, workspace, workspace_bytes, &L)) !=
+        TWINKV_OK)
+        return r;
+    DeviceInfo* dev = nullptr;
+    if ((r = device_info(&dev)) != TWINKV_OK) return r;
+    return launch_select(s, score_ret, retained_mask, budget, threshold, p, out_mask, out_swaps,
+                         out_nswaps, out_status, workspace, L, static_cast<cudaStream_t>(stream),
+                         twin_ret);
 }
 
 twinkv_status twinkv_repair_select(const double* score_ret, twinkv_shape s,

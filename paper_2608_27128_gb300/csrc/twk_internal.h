@@ -53,7 +53,13 @@ struct RepairArgs {
     int* idx0;
     uint64_t* keys1;
     int* idx1;
+    // dedup variant (twin != null): a donor is not evicted together with its twin
+    const int* twin;            // [U][N] argmax position of b_i(S0), or null
+    int* rank_of;               // [U][N] scratch: donor rank of each position
 };
+
+// Largest N the dedup variant accepts: its walk keeps 2 bits per donor in shared memory.
+constexpr int kDedupMaxN = 1 << 19;
 
 // prep kernels
 cudaError_t launch_round_bf16(const float* in, uint16_t* out, int64_t n, cudaStream_t st);

@@ -15,6 +15,16 @@
 //   5. m = min(|O|, |D|): S1 = S0 with the first m donors cleared and the first m
 //      orphans set; swaps[k] = (donor k, orphan k).
 // Sort buffers are caller workspace ([U][N] keys and positions, twice).
+//
+// Dedup variant (repair_kernel<true>, given the twin of every position): evicting a
+// donor keeps its twin, so a twin pair never loses both members.  All donors are
+// sorted; each gets the donor rank of its twin (through a position -> rank table in
+// the workspace); one thread then walks the ranks in severity order with two bits of
+// state per rank in shared memory (evicted, pinned): a donor is skipped when it is
+// pinned (the twin of an evicted donor) or its twin is evicted, and the walk stops
+// after |O| evictions.  The ranks it needs are staged in shared memory chunk by chunk,
+// so the walk itself touches shared memory only.  m = the evictions; the m most
+// severe orphans are selected as before.
 #include "twk_internal.h"
 
 namespace twk {
@@ -232,6 +242,16 @@ __device__ const int* most_severe(Shared& s, uint64_t* k, int* i, uint64_t* kx, 
     return radix_sort(s, k, i, kx, ix, n) ? ix : i;
 }
 
+constexpr int kWalkChunk = 4096;   // twin ranks staged per step of the dedup walk
+
+// Dynamic shared memory of the dedup variant: 2 state bits per donor rank (n_d <= N),
+// then one chunk of staged twin ranks.
+inline size_t dedup_smem_bytes(int N)
+{
+    return static_cast<size_t>((N + 15) / 16) * 4 + kWalkChunk * 4;
+}
+
+template <bool kDedup>
 __global__ void __launch_bounds__(kT, 1) repair_kernel(const RepairArgs a)
 {
     __shared__ Shared s;
@@ -316,12 +336,64 @@ __global__ void __launch_bounds__(kT, 1) repair_kernel(const RepairArgs a)
     __syncthreads();
 
     // 4. the m most severe orphans and donors, in severity order
-    const int* orph = most_severe(s, k0, i0, k1, i1, n_o, m);
-    const int* don = most_severe(s, k0 + n_o, i0 + n_o, k1 + n_o, i1 + n_o, n_d, m);
+    const int* orph;
+    const int* don;
+    int m_eff = m;
+    if (!kDedup) {
+        orph = most_severe(s, k0, i0, k1, i1, n_o, m);
+        don = most_severe(s, k0 + n_o, i0 + n_o, k1 + n_o, i1 + n_o, n_d, m);
+    } else {
+        extern __shared__ uint32_t dyn[];
+        uint32_t* state = dyn;                                   // 2 bits per rank
+        int* trs = reinterpret_cast<int*>(dyn + (N + 15) / 16);  // staged twin ranks
+        // every donor in severity order; the other position buffer and the key
+        // buffers' donor regions are free afterwards
+        const int* spos = most_severe(s, k0 + n_o, i0 + n_o, k1 + n_o, i1 + n_o, n_d, n_d);
+        int* tr = spos == i0 + n_o ? i1 + n_o : i0 + n_o;
+        int* dlist = reinterpret_cast<int*>(k0 + n_o);
+        int* R = a.rank_of + off;
+        for (int i = threadIdx.x; i < N; i += kT) R[i] = -1;
+        for (int w = threadIdx.x; w < (n_d + 15) / 16; w += kT) state[w] = 0;
+        __syncthreads();
+        for (int k = threadIdx.x; k < n_d; k += kT) R[spos[k]] = k;
+        __syncthreads();
+        const int* tw = a.twin + off;
+        for (int k = threadIdx.x; k < n_d; k += kT) {
+            const int t = tw[spos[k]];
+            tr[k] = (t >= 0 && t < N) ? R[t] : -1;
+        }
+        __syncthreads();
+        int acc = 0;
+        for (int c0 = 0; c0 < n_d && acc < n_o; c0 += kWalkChunk) {
+            const int len = min(kWalkChunk, n_d - c0);
+            for (int j = threadIdx.x; j < len; j += kT) trs[j] = tr[c0 + j];
+            __syncthreads();
+            if (threadIdx.x == 0) {
+                for (int j = 0; j < len && acc < n_o; ++j) {
+                    const int k = c0 + j;
+                    if ((state[k >> 4] >> ((k & 15) * 2)) & 2u) continue;          // pinned
+                    const int t = trs[j];
+                    if (t >= 0 && ((state[t >> 4] >> ((t & 15) * 2)) & 1u)) continue;  // twin out
+                    state[k >> 4] |= 1u << ((k & 15) * 2);
+                    if (t >= 0) state[t >> 4] |= 2u << ((t & 15) * 2);
+                    dlist[acc++] = k;
+                }
+                s.flag = acc;
+            }
+            __syncthreads();
+            acc = s.flag;
+            __syncthreads();
+        }
+        m_eff = acc;
+        for (int j = threadIdx.x; j < m_eff; j += kT) dlist[j] = spos[dlist[j]];
+        __syncthreads();
+        orph = most_severe(s, k0, i0, k1, i1, n_o, m_eff);
+        don = dlist;
+    }
     __syncthreads();
 
     // 5. swap
-    for (int k = threadIdx.x; k < m; k += kT) {
+    for (int k = threadIdx.x; k < m_eff; k += kT) {
         const int out_ = don[k], in_ = orph[k];
         S1[out_] = 0;
         S1[in_] = 1;
@@ -329,7 +401,7 @@ __global__ void __launch_bounds__(kT, 1) repair_kernel(const RepairArgs a)
         swaps[2 * k + 1] = in_;
     }
     if (threadIdx.x == 0) {
-        a.out_nswaps[u] = m;
+        a.out_nswaps[u] = m_eff;
         if (a.out_status) a.out_status[u] = 0;
     }
 }
@@ -338,7 +410,16 @@ __global__ void __launch_bounds__(kT, 1) repair_kernel(const RepairArgs a)
 
 cudaError_t launch_repair(const RepairArgs& a, cudaStream_t st)
 {
-    repair_kernel<<<a.U, kT, 0, st>>>(a);
+    if (!a.twin) {
+        repair_kernel<false><<<a.U, kT, 0, st>>>(a);
+        return cudaGetLastError();
+    }
+    if (a.N > kDedupMaxN) return cudaErrorInvalidValue;
+    const size_t bytes = dedup_smem_bytes(a.N);
+    const cudaError_t e = cudaFuncSetAttribute(
+        repair_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(bytes));
+    if (e != cudaSuccess) return e;
+    repair_kernel<true><<<a.U, kT, bytes, st>>>(a);
     return cudaGetLastError();
 }
 

@@ -23,7 +23,7 @@ from . import build as _build
  ERR_TOO_LARGE) = range(8)
 NOALLOC_MAX_POSITIONS = 262144
 BF16, F32 = 0, 1
-OP_REDUNDANCY, OP_REPAIR, OP_REPAIR_SELECT, OP_POLICY = 0, 1, 2, 3
+OP_REDUNDANCY, OP_REPAIR, OP_REPAIR_SELECT, OP_POLICY, OP_REPAIR_SELECT_DEDUP = 0, 1, 2, 3, 4
 KERNEL_PREP, KERNEL_AUDIT, KERNEL_REPAIR, KERNEL_REFINE = 0, 1, 2, 3
 KERNEL_NAMES = ("prep", "audit", "repair", "refine")
 
@@ -33,7 +33,7 @@ EXPORTED = (
     "twinkv_status_string", "twinkv_get_last_error", "twinkv_set_wait_timeout_ns",
     "twinkv_wait_probe", "twinkv_profile_begin", "twinkv_profile_end",
     "twinkv_repair_select_noalloc", "twinkv_host_arena_size", "twinkv_repair_host",
-    "twinkv_policy",
+    "twinkv_policy", "twinkv_repair_dedup", "twinkv_repair_select_dedup",
 )
 
 
@@ -97,6 +97,10 @@ def load(build_if_missing: bool = True):
         lib.twinkv_repair_host.argtypes = [_P, Shape, _P, _P, ctypes.c_float,
                                            ctypes.POINTER(Params), _P, _P, _P, _P, _P, _P, _P,
                                            _P, ctypes.c_int32, _P, ctypes.c_size_t, _P]
+        lib.twinkv_repair_dedup.argtypes = lib.twinkv_repair.argtypes
+        lib.twinkv_repair_select_dedup.argtypes = [_P, _P, Shape, _P, _P, ctypes.c_float,
+                                                   ctypes.POINTER(Params), _P, _P, _P, _P, _P,
+                                                   ctypes.c_size_t, _P]
         lib.twinkv_policy.argtypes = [_P, Shape, _P, ctypes.c_float, ctypes.POINTER(Params),
                                       _P, _P, _P, _P, ctypes.c_size_t, _P]
         lib.twinkv_status_string.argtypes = [ctypes.c_int]
@@ -107,6 +111,7 @@ def load(build_if_missing: bool = True):
                                            ctypes.POINTER(ctypes.c_double)]
         for name in ("twinkv_redundancy", "twinkv_repair", "twinkv_repair_select",
                      "twinkv_repair_select_noalloc", "twinkv_repair_host", "twinkv_policy",
+                     "twinkv_repair_dedup", "twinkv_repair_select_dedup",
                      "twinkv_get_last_error", "twinkv_set_wait_timeout_ns",
                      "twinkv_wait_probe", "twinkv_profile_begin", "twinkv_profile_end"):
             getattr(lib, name).restype = ctypes.c_int
@@ -229,9 +234,17 @@ def _params(params, threshold, window, n_sink, n_recent):
     return p
 
 
+def twinkv_repair_dedup(keys, retained_mask, budget=None, threshold=None, params=None,
+                        **kw) -> dict:
+    """twinkv_repair, but a donor is never evicted together with its twin (see the C
+    header); same arguments and outputs."""
+    return twinkv_repair(keys, retained_mask, budget, threshold, params, _fn="twinkv_repair_dedup",
+                         **kw)
+
+
 def twinkv_repair(keys, retained_mask, budget=None, threshold=None, params=None, *,
                   window=None, n_sink=None, n_recent=None, want_ret=True, want_all=False,
-                  out=None, ws=None, stream=None) -> dict:
+                  out=None, ws=None, stream=None, _fn="twinkv_repair") -> dict:
     """Audit of the retained set S0 and the budget-exact orphan/donor swap.
 
     keys [L,H,N,d] bf16/float32; retained_mask [L,H,N] uint8; budget [L*H] int32 or None.
@@ -261,12 +274,43 @@ def twinkv_repair(keys, retained_mask, budget=None, threshold=None, params=None,
         o["score_all"] = _out(out.get("score_all"), "score_all", torch.float64, (L, H, N), dev)
         o["twin_all"] = _out(out.get("twin_all"), "twin_all", torch.int32, (L, H, N), dev)
     ws = _ws(ws, s, OP_REPAIR, dev)
-    st = load().twinkv_repair(
+    st = getattr(load(), _fn)(
         _ptr(keys), s, _ptr(retained_mask), _ptr(budget), ctypes.c_float(p.threshold),
         ctypes.byref(p), _ptr(o["mask"]), _ptr(o["swaps"]), _ptr(o["nswaps"]),
         _ptr(o.get("score_ret")), _ptr(o.get("twin_ret")), _ptr(o.get("score_all")),
         _ptr(o.get("twin_all")), _ptr(o["status"]), _ptr(ws), ws.numel(), _stream(stream))
-    _check(st, "twinkv_repair")
+    _check(st, _fn)
+    return o
+
+
+def twinkv_repair_select_dedup(score_ret, twin_ret, retained_mask, budget=None, threshold=None,
+                               params=None, *, n_sink=None, n_recent=None, out=None, ws=None,
+                               stream=None) -> dict:
+    """The dedup selection alone, on given float64 b_i(S0) and int32 twins [L,H,N]."""
+    if score_ret.dim() != 3:
+        raise ValueError("score_ret must be [L, H, N]")
+    L, H, N = (int(x) for x in score_ret.shape)
+    dev = score_ret.device
+    _need(score_ret, "score_ret", torch.float64, (L, H, N), dev)
+    _need(twin_ret, "twin_ret", torch.int32, (L, H, N), dev)
+    _need(retained_mask, "retained_mask", torch.uint8, (L, H, N), dev)
+    if budget is not None:
+        _need(budget, "budget", torch.int32, (L * H,), dev)
+    s = Shape(L, H, N, 64, BF16)
+    p = _params(params, threshold, None, n_sink, n_recent)
+    out = dict(out or {})
+    o = {
+        "mask": _out(out.get("mask"), "mask", torch.uint8, (L, H, N), dev),
+        "swaps": _out(out.get("swaps"), "swaps", torch.int32, (L * H, N // 2, 2), dev),
+        "nswaps": _out(out.get("nswaps"), "nswaps", torch.int32, (L * H,), dev),
+        "status": _out(out.get("status"), "status", torch.int32, (L * H,), dev),
+    }
+    ws = _ws(ws, s, OP_REPAIR_SELECT_DEDUP, dev)
+    st = load().twinkv_repair_select_dedup(
+        _ptr(score_ret), _ptr(twin_ret), s, _ptr(retained_mask), _ptr(budget),
+        ctypes.c_float(p.threshold), ctypes.byref(p), _ptr(o["mask"]), _ptr(o["swaps"]),
+        _ptr(o["nswaps"]), _ptr(o["status"]), _ptr(ws), ws.numel(), _stream(stream))
+    _check(st, "twinkv_repair_select_dedup")
     return o
 
 
