@@ -297,18 +297,23 @@ def run_e2e(args, world, w, keys_h, mask_h, budget_h, out, stream):
         res = tk.twinkv_repair_host(keys_p, mask_p, budget_p, threshold=w.tau, want_all=True,
                                     chunk_units=chunk, out=res, arena=arena, stream=stream)
 
-    for _ in range(2):
+    for _ in range(max(2, args.warmup)):
         e2e_step()
     torch.cuda.synchronize()
-    e2e_steps = max(3, args.steps // 2)
+    e2e_steps = max(3, args.steps)
     barrier(world)
-    f0, f1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    f0.record(stream)
-    for _ in range(e2e_steps):
+    # one event between consecutive steps: the mean over all steps is the reported
+    # value; the per-step median and maximum show whether a few slow steps moved it
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(e2e_steps + 1)]
+    ev[0].record(stream)
+    for k in range(e2e_steps):
         e2e_step()
-    f1.record(stream)
+        ev[k + 1].record(stream)
     torch.cuda.synchronize()
-    e2e_ms = max_over_ranks(f0.elapsed_time(f1) / e2e_steps, world)
+    e2e_ms = max_over_ranks(ev[0].elapsed_time(ev[-1]) / e2e_steps, world)
+    per_step = [ev[k].elapsed_time(ev[k + 1]) for k in range(e2e_steps)]
+    args.e2e_step_stats = {"steps": e2e_steps, "ms_median": statistics.median(per_step),
+                           "ms_max": max(per_step), "ms_min": min(per_step)}
     assert tk.twinkv_get_last_error() == tk.OK
     # the step's results match the device-resident run
     for k in ("mask", "nswaps", "score_all", "twin_ret"):
@@ -354,7 +359,8 @@ def _report(args, w, ratio, world, U, N, d, ms, prof, e2e_ms, h2d, d2h, chunk, c
         "e2e": None if e2e_ms is None else {
             "value": job_throughput(world, U * N, e2e_ms), "unit": "keys/s",
             "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms,
-            "api": "twinkv_repair_host", "chunk_units": chunk},
+            "api": "twinkv_repair_host", "chunk_units": chunk,
+            **getattr(args, "e2e_step_stats", {})},
         "clocks": clocks.summary(),
     }
     if not args.no_cpu:

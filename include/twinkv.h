@@ -218,16 +218,19 @@ twinkv_status twinkv_repair_select_noalloc(const double* score_ret, twinkv_shape
  * twinkv_repair on a cache held in host memory (for example a KV cache offloaded to the
  * host): the same audit and swap (Sec. 3.4), with every tensor argument a HOST pointer
  * of the layout above (page-locked memory lets the copies run asynchronously).  The
- * units are processed in chunks of `chunk_units` units (0: a quarter of L*H): chunk
- * c + 1 is copied to the device while chunk c is computed on `stream`, and results are
- * copied back while later chunks run, so the copies hide behind the computation.
+ * units' keys go to the device in chunks of `chunk_units` units (0: a quarter of L*H):
+ * chunk c + 1 is copied in while the audit of chunk c runs on `stream`, and each
+ * chunk's scores and twins are copied back while later chunks run.  One selection over
+ * all units follows the last chunk, and S1, the swap lists, counts and statuses are
+ * copied back after it.
  *   arena        caller-owned DEVICE memory of twinkv_host_arena_size(s, chunk_units)
- *                bytes, 256-byte aligned: double-buffered chunk inputs and outputs plus
- *                one chunk's workspace.  The library allocates nothing.
+ *                bytes, 256-byte aligned: two chunk buffers of keys, the mask, b and
+ *                twins of every unit, the outputs, one chunk's workspace and the
+ *                selection's workspace.  The library allocates nothing.
  *   out_*        host outputs as in twinkv_repair (out_score_ret .. out_twin_all may be
  *                NULL); valid once `stream` has completed.  Unlike twinkv_repair, the
  *                entries of out_swaps past out_nswaps[u] are overwritten with
- *                unspecified values (whole chunks are copied back).
+ *                unspecified values (the whole swap array is copied back).
  * The copies run on two streams the library keeps per device; calls on one device are
  * ordered after each other's use of the arena.
  */

@@ -285,12 +285,15 @@ bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 
 int default_chunk_units(int U) { return U < 4 ? U : (U + 3) / 4; }
 
 struct HostArena {
-    size_t keys = 0, mask = 0, budget = 0, omask = 0, oswaps = 0, onswaps = 0, ostatus = 0,
-           osret = 0, otret = 0, osall = 0, otall = 0;
-    size_t per_buf = 0, ws = 0, ws_bytes = 0, total = 0;
+    // keys: two chunk buffers; every other array covers all units
+    size_t keys = 0, mask = 0, budget = 0, bret = 0, tret = 0, sall = 0, tall = 0, omask = 0,
+           oswaps = 0, onswaps = 0, ostatus = 0;
+    size_t key_buf = 0;                // bytes of one keys chunk buffer
+    size_t ws = 0, ws_bytes = 0;       // audit-stage workspace of one chunk
+    size_t sel = 0, sel_bytes = 0;     // selection workspace over all units
+    size_t total = 0;
 };
 
-// One chunk's inputs and outputs (twice, for double buffering) and one workspace.
 HostArena host_arena(const twinkv_shape& s, int uc)
 {
     HostArena A;
@@ -300,33 +303,35 @@ HostArena host_arena(const twinkv_shape& s, int uc)
         off += up256(bytes);
         return o;
     };
-    const size_t N = static_cast<size_t>(s.N), U = static_cast<size_t>(uc);
+    const size_t N = static_cast<size_t>(s.N), U = static_cast<size_t>(s.L) * s.H;
     const size_t esize = s.dtype == TWINKV_F32 ? 4 : 2;
-    A.keys = take(U * N * s.d * esize);
+    A.key_buf = up256(static_cast<size_t>(uc) * N * s.d * esize);
+    A.keys = take(2 * A.key_buf);
     A.mask = take(U * N);
     A.budget = take(U * 4);
+    A.bret = take(U * N * 8);
+    A.tret = take(U * N * 4);
+    A.sall = take(U * N * 8);
+    A.tall = take(U * N * 4);
     A.omask = take(U * N);
     A.oswaps = take(U * (N / 2) * 2 * 4);
     A.onswaps = take(U * 4);
     A.ostatus = take(U * 4);
-    A.osret = take(U * N * 8);
-    A.otret = take(U * N * 4);
-    A.osall = take(U * N * 8);
-    A.otall = take(U * N * 4);
-    A.per_buf = off;
     twinkv_shape sc = s;
     sc.L = 1;
     sc.H = uc;
-    A.ws = 2 * A.per_buf;
     A.ws_bytes = layout(sc, TWINKV_OP_REPAIR).total;
-    A.total = A.ws + A.ws_bytes;
+    A.ws = take(A.ws_bytes);
+    A.sel_bytes = layout(s, TWINKV_OP_REPAIR_SELECT).total;
+    A.sel = take(A.sel_bytes);
+    A.total = off;
     return A;
 }
 
 struct HostStreams {
     bool ready = false;
     cudaStream_t h2d = nullptr, d2h = nullptr;
-    cudaEvent_t in[2], done[2], out[2];
+    cudaEvent_t in[2], done[2], sel, fin;
 };
 HostStreams g_hs[kMaxDevices];
 
@@ -342,9 +347,11 @@ twinkv_status host_streams(HostStreams** out)
             return TWINKV_ERR_CUDA;
         for (int b = 0; b < 2; ++b)
             if (cudaEventCreateWithFlags(&h.in[b], cudaEventDisableTiming) != cudaSuccess ||
-                cudaEventCreateWithFlags(&h.done[b], cudaEventDisableTiming) != cudaSuccess ||
-                cudaEventCreateWithFlags(&h.out[b], cudaEventDisableTiming) != cudaSuccess)
+                cudaEventCreateWithFlags(&h.done[b], cudaEventDisableTiming) != cudaSuccess)
                 return TWINKV_ERR_CUDA;
+        if (cudaEventCreateWithFlags(&h.sel, cudaEventDisableTiming) != cudaSuccess ||
+            cudaEventCreateWithFlags(&h.fin, cudaEventDisableTiming) != cudaSuccess)
+            return TWINKV_ERR_CUDA;
         h.ready = true;
     }
     *out = &h;
@@ -614,25 +621,15 @@ twinkv_status twinkv_policy(const void* keys, twinkv_shape s, const int32_t* bud
 }  // extern "C"
 
 namespace {
-twinkv_status repair_impl(const void* keys, twinkv_shape s, const uint8_t* retained_mask,
-                          const int32_t* budget, float threshold, const twinkv_params* params,
-                          uint8_t* out_mask, int32_t* out_swaps, int32_t* out_nswaps,
-                          double* out_score_ret, int32_t* out_twin_ret, double* out_score_all,
-                          int32_t* out_twin_all, int32_t* out_status, void* workspace,
-                          size_t workspace_bytes, void* stream, bool dedup)
+// The audit stages of the repair for one set of units: bf16 keys, retained-first
+// gather, audit, exact values.  Writes b_i(S0) to bret and its twin's position to t0;
+// b_i(all) and its twin to out_score_all / out_twin_all when either is given.
+twinkv_status audit_stages(const DeviceInfo* dev, const void* keys, const twinkv_shape& s,
+                           const uint8_t* retained_mask, const twinkv_params& p, double* bret,
+                           int* t0, double* out_score_all, int32_t* out_twin_all,
+                           void* workspace, const Layout& L, cudaStream_t st)
 {
-    const twinkv_params p = params ? *params : twinkv_default_params();
-    if (!keys || !aligned16(keys) || !retained_mask || !out_mask || !out_nswaps ||
-        !shape_ok(s, true) || (!out_swaps && s.N >= 2))   // with N < 2 no swap fits
-        return TWINKV_ERR_INVALID_ARG;
-    twinkv_status r = params_ok(p, threshold);
-    if (r != TWINKV_OK) return r;
-    Layout L;
-    if ((r = check_ws(s, TWINKV_OP_REPAIR, workspace, workspace_bytes, &L)) != TWINKV_OK) return r;
-    DeviceInfo* dev = nullptr;
-    if ((r = device_info(&dev)) != TWINKV_OK) return r;
-    cudaStream_t st = static_cast<cudaStream_t>(stream);
-
+    twinkv_status r;
     const uint16_t* k16 = nullptr;
     if ((r = keys_bf16(keys, s, workspace, L, st, &k16)) != TWINKV_OK) return r;
     const int U = s.L * s.H;
@@ -654,9 +651,7 @@ twinkv_status repair_impl(const void* keys, twinkv_shape s, const uint8_t* retai
             return TWINKV_ERR_CUDA;
     }
     const bool need_all = out_score_all || out_twin_all;
-    int* t0 = out_twin_ret ? out_twin_ret : at<int>(workspace, L.twin0);
     int* t1 = need_all ? (out_twin_all ? out_twin_all : at<int>(workspace, L.twin1)) : nullptr;
-    double* bret = out_score_ret ? out_score_ret : at<double>(workspace, L.bret);
     AuditArgs a;
     std::memset(&a, 0, sizeof a);
     a.U = U;
@@ -678,7 +673,32 @@ twinkv_status repair_impl(const void* keys, twinkv_shape s, const uint8_t* retai
     a.mant_mask = 0xFFFFFFE0u;
     if ((r = run_audit(*dev, s, k16, kp, static_cast<int64_t>(U) * NP, a, st)) != TWINKV_OK)
         return r;
-    if ((r = run_refine(k16, s, norm2, t0, t1, bret, out_score_all, st)) != TWINKV_OK)
+    return run_refine(k16, s, norm2, t0, t1, bret, out_score_all, st);
+}
+
+twinkv_status repair_impl(const void* keys, twinkv_shape s, const uint8_t* retained_mask,
+                          const int32_t* budget, float threshold, const twinkv_params* params,
+                          uint8_t* out_mask, int32_t* out_swaps, int32_t* out_nswaps,
+                          double* out_score_ret, int32_t* out_twin_ret, double* out_score_all,
+                          int32_t* out_twin_all, int32_t* out_status, void* workspace,
+                          size_t workspace_bytes, void* stream, bool dedup)
+{
+    const twinkv_params p = params ? *params : twinkv_default_params();
+    if (!keys || !aligned16(keys) || !retained_mask || !out_mask || !out_nswaps ||
+        !shape_ok(s, true) || (!out_swaps && s.N >= 2))   // with N < 2 no swap fits
+        return TWINKV_ERR_INVALID_ARG;
+    twinkv_status r = params_ok(p, threshold);
+    if (r != TWINKV_OK) return r;
+    Layout L;
+    if ((r = check_ws(s, TWINKV_OP_REPAIR, workspace, workspace_bytes, &L)) != TWINKV_OK) return r;
+    DeviceInfo* dev = nullptr;
+    if ((r = device_info(&dev)) != TWINKV_OK) return r;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+
+    int* t0 = out_twin_ret ? out_twin_ret : at<int>(workspace, L.twin0);
+    double* bret = out_score_ret ? out_score_ret : at<double>(workspace, L.bret);
+    if ((r = audit_stages(dev, keys, s, retained_mask, p, bret, t0, out_score_all,
+                          out_twin_all, workspace, L, st)) != TWINKV_OK)
         return r;
     return launch_select(s, bret, retained_mask, budget, threshold, p, out_mask, out_swaps,
                          out_nswaps, out_status, workspace, L, st, dedup ? t0 : nullptr);
@@ -823,71 +843,77 @@ twinkv_status twinkv_repair_host(const void* keys, twinkv_shape s, const uint8_t
     char* base = static_cast<char*>(arena);
     const size_t N = static_cast<size_t>(s.N);
     const size_t esize = s.dtype == TWINKV_F32 ? 4 : 2;
-    const size_t swaps_per_unit = (N / 2) * 2;
     auto ck = [&](cudaError_t e) { return e == cudaSuccess; };
-    // The previous call's last uses of both buffers come first.
-    for (int b = 0; b < 2; ++b) {
-        if (!ck(cudaStreamWaitEvent(hs->h2d, hs->done[b], 0)) ||
-            !ck(cudaStreamWaitEvent(hs->h2d, hs->out[b], 0)) ||
-            !ck(cudaStreamWaitEvent(st, hs->out[b], 0)))
-            return TWINKV_ERR_CUDA;
-    }
+    uint8_t* d_mask = reinterpret_cast<uint8_t*>(base + A.mask);
+    int32_t* d_budget = budget ? reinterpret_cast<int32_t*>(base + A.budget) : nullptr;
+    double* d_bret = reinterpret_cast<double*>(base + A.bret);
+    int32_t* d_tret = reinterpret_cast<int32_t*>(base + A.tret);
+    double* d_sall = reinterpret_cast<double*>(base + A.sall);
+    int32_t* d_tall = reinterpret_cast<int32_t*>(base + A.tall);
+    const bool need_all = out_score_all || out_twin_all;
+    // A previous call's copies and selection finish before this call reuses the arena.
+    if (!ck(cudaStreamWaitEvent(hs->h2d, hs->fin, 0)) || !ck(cudaStreamWaitEvent(st, hs->fin, 0)))
+        return TWINKV_ERR_CUDA;
+    if (budget && !ck(cudaMemcpyAsync(d_budget, budget, U * 4, cudaMemcpyHostToDevice, hs->h2d)))
+        return TWINKV_ERR_CUDA;
     const int nchunks = (U + uc - 1) / uc;
     for (int c = 0; c < nchunks; ++c) {
         const int b = c & 1;
         const size_t u0 = static_cast<size_t>(c) * uc;
         const int un = static_cast<int>(U - u0 < static_cast<size_t>(uc) ? U - u0 : uc);
-        char* buf = base + b * A.per_buf;
-        // inputs, once the compute that last read this buffer is done
+        char* kbuf = base + A.keys + b * A.key_buf;
+        // inputs, once the audit that last read this keys buffer is done
         if (c >= 2 && !ck(cudaStreamWaitEvent(hs->h2d, hs->done[b], 0))) return TWINKV_ERR_CUDA;
-        if (!ck(cudaMemcpyAsync(buf + A.keys, static_cast<const char*>(keys) + u0 * N * s.d * esize,
+        if (!ck(cudaMemcpyAsync(kbuf, static_cast<const char*>(keys) + u0 * N * s.d * esize,
                                 un * N * s.d * esize, cudaMemcpyHostToDevice, hs->h2d)) ||
-            !ck(cudaMemcpyAsync(buf + A.mask, retained_mask + u0 * N, un * N,
+            !ck(cudaMemcpyAsync(d_mask + u0 * N, retained_mask + u0 * N, un * N,
                                 cudaMemcpyHostToDevice, hs->h2d)) ||
-            (budget && !ck(cudaMemcpyAsync(buf + A.budget, budget + u0, un * 4,
-                                           cudaMemcpyHostToDevice, hs->h2d))) ||
             !ck(cudaEventRecord(hs->in[b], hs->h2d)))
             return TWINKV_ERR_CUDA;
-        // compute on the caller's stream, once the inputs landed and this buffer's
-        // previous outputs were copied out
+        // the audit stages of this chunk, into the all-unit arrays
         if (!ck(cudaStreamWaitEvent(st, hs->in[b], 0))) return TWINKV_ERR_CUDA;
-        if (c >= 2 && !ck(cudaStreamWaitEvent(st, hs->out[b], 0))) return TWINKV_ERR_CUDA;
         twinkv_shape sc = s;
         sc.L = 1;
         sc.H = un;
-        r = twinkv_repair(buf + A.keys, sc, reinterpret_cast<const uint8_t*>(buf + A.mask),
-                          budget ? reinterpret_cast<const int32_t*>(buf + A.budget) : nullptr,
-                          threshold, &p, reinterpret_cast<uint8_t*>(buf + A.omask),
-                          reinterpret_cast<int32_t*>(buf + A.oswaps),
-                          reinterpret_cast<int32_t*>(buf + A.onswaps),
-                          out_score_ret ? reinterpret_cast<double*>(buf + A.osret) : nullptr,
-                          out_twin_ret ? reinterpret_cast<int32_t*>(buf + A.otret) : nullptr,
-                          out_score_all ? reinterpret_cast<double*>(buf + A.osall) : nullptr,
-                          out_twin_all ? reinterpret_cast<int32_t*>(buf + A.otall) : nullptr,
-                          reinterpret_cast<int32_t*>(buf + A.ostatus), base + A.ws, A.ws_bytes,
-                          st);
+        const Layout Lc = layout(sc, TWINKV_OP_REPAIR);
+        r = audit_stages(dev, kbuf, sc, d_mask + u0 * N, p, d_bret + u0 * N, d_tret + u0 * N,
+                         need_all ? d_sall + u0 * N : nullptr, need_all ? d_tall + u0 * N : nullptr,
+                         base + A.ws, Lc, st);
         if (r != TWINKV_OK) return r;
         if (!ck(cudaEventRecord(hs->done[b], st))) return TWINKV_ERR_CUDA;
-        // outputs
+        // this chunk's scores and twins go back while later chunks run
         if (!ck(cudaStreamWaitEvent(hs->d2h, hs->done[b], 0))) return TWINKV_ERR_CUDA;
-        auto d2h = [&](void* dst, size_t off, size_t bytes) {
-            return ck(cudaMemcpyAsync(dst, buf + off, bytes, cudaMemcpyDeviceToHost, hs->d2h));
+        auto d2h = [&](void* dst, const void* src, size_t bytes) {
+            return ck(cudaMemcpyAsync(dst, src, bytes, cudaMemcpyDeviceToHost, hs->d2h));
         };
-        if (!d2h(out_mask + u0 * N, A.omask, un * N) ||
-            (out_swaps && !d2h(out_swaps + u0 * swaps_per_unit, A.oswaps,
-                               un * swaps_per_unit * 4)) ||
-            !d2h(out_nswaps + u0, A.onswaps, un * 4) ||
-            (out_status && !d2h(out_status + u0, A.ostatus, un * 4)) ||
-            (out_score_ret && !d2h(out_score_ret + u0 * N, A.osret, un * N * 8)) ||
-            (out_twin_ret && !d2h(out_twin_ret + u0 * N, A.otret, un * N * 4)) ||
-            (out_score_all && !d2h(out_score_all + u0 * N, A.osall, un * N * 8)) ||
-            (out_twin_all && !d2h(out_twin_all + u0 * N, A.otall, un * N * 4)) ||
-            !ck(cudaEventRecord(hs->out[b], hs->d2h)))
+        if ((out_score_ret && !d2h(out_score_ret + u0 * N, d_bret + u0 * N, un * N * 8)) ||
+            (out_twin_ret && !d2h(out_twin_ret + u0 * N, d_tret + u0 * N, un * N * 4)) ||
+            (out_score_all && !d2h(out_score_all + u0 * N, d_sall + u0 * N, un * N * 8)) ||
+            (out_twin_all && !d2h(out_twin_all + u0 * N, d_tall + u0 * N, un * N * 4)))
             return TWINKV_ERR_CUDA;
     }
-    // The caller's stream completes only after the last results reached the host.
-    for (int b = 0; b < 2; ++b)
-        if (!ck(cudaStreamWaitEvent(st, hs->out[b], 0))) return TWINKV_ERR_CUDA;
+    // one selection over every unit (Sec. 3.4), then its results go back
+    const Layout Lsel = layout(s, TWINKV_OP_REPAIR_SELECT);
+    uint8_t* d_omask = reinterpret_cast<uint8_t*>(base + A.omask);
+    int32_t* d_oswaps = reinterpret_cast<int32_t*>(base + A.oswaps);
+    int32_t* d_onswaps = reinterpret_cast<int32_t*>(base + A.onswaps);
+    int32_t* d_ostatus = reinterpret_cast<int32_t*>(base + A.ostatus);
+    if ((r = launch_select(s, d_bret, d_mask, d_budget, threshold, p, d_omask, d_oswaps,
+                           d_onswaps, d_ostatus, base + A.sel, Lsel, st)) != TWINKV_OK)
+        return r;
+    if (!ck(cudaEventRecord(hs->sel, st)) || !ck(cudaStreamWaitEvent(hs->d2h, hs->sel, 0)))
+        return TWINKV_ERR_CUDA;
+    const size_t swaps_bytes = static_cast<size_t>(U) * (N / 2) * 2 * 4;
+    if (!ck(cudaMemcpyAsync(out_mask, d_omask, U * N, cudaMemcpyDeviceToHost, hs->d2h)) ||
+        (out_swaps && swaps_bytes &&
+         !ck(cudaMemcpyAsync(out_swaps, d_oswaps, swaps_bytes, cudaMemcpyDeviceToHost, hs->d2h))) ||
+        !ck(cudaMemcpyAsync(out_nswaps, d_onswaps, U * 4, cudaMemcpyDeviceToHost, hs->d2h)) ||
+        (out_status &&
+         !ck(cudaMemcpyAsync(out_status, d_ostatus, U * 4, cudaMemcpyDeviceToHost, hs->d2h))) ||
+        !ck(cudaEventRecord(hs->fin, hs->d2h)))
+        return TWINKV_ERR_CUDA;
+    // The caller's stream completes only after the results reached the host.
+    if (!ck(cudaStreamWaitEvent(st, hs->fin, 0))) return TWINKV_ERR_CUDA;
     return TWINKV_OK;
 }
 
