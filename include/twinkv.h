@@ -218,7 +218,8 @@ twinkv_status twinkv_repair_select_noalloc(const double* score_ret, twinkv_shape
  * twinkv_repair on a cache held in host memory (for example a KV cache offloaded to the
  * host): the same audit and swap (Sec. 3.4), with every tensor argument a HOST pointer
  * of the layout above (page-locked memory lets the copies run asynchronously).  The
- * units' keys go to the device in chunks of `chunk_units` units (0: a quarter of L*H):
+ * units' keys go to the device in chunks of `chunk_units` units (0: a quarter of L*H;
+ * the first chunk is a quarter of that, since nothing computes while it copies in):
  * chunk c + 1 is copied in while the audit of chunk c runs on `stream`, and each
  * chunk's scores and twins are copied back while later chunks run.  One selection over
  * all units follows the last chunk, and S1, the swap lists, counts and statuses are

@@ -856,11 +856,13 @@ twinkv_status twinkv_repair_host(const void* keys, twinkv_shape s, const uint8_t
         return TWINKV_ERR_CUDA;
     if (budget && !ck(cudaMemcpyAsync(d_budget, budget, U * 4, cudaMemcpyHostToDevice, hs->h2d)))
         return TWINKV_ERR_CUDA;
-    const int nchunks = (U + uc - 1) / uc;
-    for (int c = 0; c < nchunks; ++c) {
+    // The first chunk is a quarter of the others: nothing computes while it copies in.
+    const int first = uc >= 4 ? uc / 4 : uc;
+    size_t u0 = 0;
+    for (int c = 0; u0 < static_cast<size_t>(U); ++c) {
         const int b = c & 1;
-        const size_t u0 = static_cast<size_t>(c) * uc;
-        const int un = static_cast<int>(U - u0 < static_cast<size_t>(uc) ? U - u0 : uc);
+        const int want = c == 0 ? first : uc;
+        const int un = static_cast<int>(U - u0 < static_cast<size_t>(want) ? U - u0 : want);
         char* kbuf = base + A.keys + b * A.key_buf;
         // inputs, once the audit that last read this keys buffer is done
         if (c >= 2 && !ck(cudaStreamWaitEvent(hs->h2d, hs->done[b], 0))) return TWINKV_ERR_CUDA;
@@ -891,6 +893,7 @@ twinkv_status twinkv_repair_host(const void* keys, twinkv_shape s, const uint8_t
             (out_score_all && !d2h(out_score_all + u0 * N, d_sall + u0 * N, un * N * 8)) ||
             (out_twin_all && !d2h(out_twin_all + u0 * N, d_tall + u0 * N, un * N * 4)))
             return TWINKV_ERR_CUDA;
+        u0 += un;
     }
     // one selection over every unit (Sec. 3.4), then its results go back
     const Layout Lsel = layout(s, TWINKV_OP_REPAIR_SELECT);
