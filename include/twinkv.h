@@ -297,10 +297,10 @@ twinkv_status twinkv_repair_select_dedup(const double* score_ret, const int32_t*
  *   out_count   [L][H][N] int32: r_i, or NULL (then kept in the workspace)
  *   out_status  [L*H] int32: 0, or TWINKV_ERR_INVALID_ARG where budget[u] is outside
  *               [0, N] (that unit's mask is all 0); or NULL
- * Precision: each pair is decided as the sign of one fp32 fused multiply-add,
- * x_ij * (1/||k_j||) - tau * ||k_i||, x_ij the fp32 tensor-core dot product of the bf16
- * keys: pairs whose similarity is within about 1e-6 of tau may count differently
- * than in exact arithmetic.
+ * Precision: each pair is decided by one fp32 fused multiply-add on the unrounded
+ * product, x_ij * (1/||k_j||) - tau * ||k_i||, x_ij the fp32 tensor-core dot product of
+ * the bf16 keys: pairs whose similarity is within about 1e-6 of tau may count
+ * differently than in exact arithmetic.
  * Workspace: twinkv_workspace_size(s, TWINKV_OP_POLICY) bytes, 256-byte aligned.
  */
 twinkv_status twinkv_policy(const void* keys, twinkv_shape s, const int32_t* budget,

@@ -589,7 +589,8 @@ twinkv_status twinkv_policy(const void* keys, twinkv_shape s, const int32_t* bud
     int* count = out_count ? out_count : at<int>(workspace, L.rcount);
     {
         ProfScope pr(TWINKV_KERNEL_PREP, st);
-        if (launch_norms_identity(k16, U, s.N, s.d, NP, colrinv, colpos, norm2, st) !=
+        if (launch_norms_identity(k16, U, s.N, s.d, NP, colrinv, colpos, norm2, st,
+                                  kCountScale) !=
             cudaSuccess)
             return TWINKV_ERR_CUDA;
     }

@@ -29,9 +29,13 @@
 //
 // Count mode (Sec. 3.2 Eq. 2, the standalone scorer): instead of the maximum, each row i
 // counts the columns j outside the window with sim(i,j) > tau.  With x_ij the raw dot
-// product, that is x_ij * (1/||k_j||) > tau * ||k_i||, evaluated as the sign of one
-// fused multiply-add x_ij * (1/||k_j||) - tau / (1/||k_i||), so the product is never
-// rounded before the comparison; masked and padding columns are NaN and never count.
+// product, that is x_ij * (1/||k_j||) > tau * ||k_i||.  The column scales arrive
+// multiplied by S = 2^32 (exact), so one fused multiply-add with saturation,
+// sat(x_ij * S/||k_j|| - S tau ||k_i||), is 1 when the pair counts and 0 when it does
+// not (NaN, for masked and padding columns, saturates to 0); only a pair within
+// 2^-32 of the threshold could give a fraction.  The product is never rounded before
+// the comparison, the count accumulates in fp32 (exact below 2^24), and all of it
+// runs on the FMA pipe.
 //
 // Column layout: in repair mode the columns of a unit are stored retained-first
 // (retained keys in position order, padded to a tile, then evicted keys in position
@@ -199,52 +203,51 @@ __device__ __forceinline__ void reduce_group(const uint32_t (&x0)[32], const uin
     fold32<kMasked>(x3, rinv + 96, pos + 96, rw, w2, mask, col0 + 96, b);
 }
 
-// 1 where a > b (false for NaN), as an all-ones word so that three-input integer adds
-// accumulate two comparisons per instruction.
-__device__ __forceinline__ uint32_t gt_mask(float a, float b)
+// sat(a * b + c): fp32 fused multiply-add clamped to [0, 1], NaN to 0.
+__device__ __forceinline__ float fma_sat(float a, float b, float c)
 {
-    uint32_t r;
-    asm("set.gt.u32.f32 %0, %1, %2;" : "=r"(r) : "f"(a), "f"(b));
+    float r;
+    asm("fma.rn.sat.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(a), "f"(b), "f"(c));
     return r;
 }
 
-// Eq. 2 over 32 columns: how many x_j / ||k_j|| exceed t = tau * ||k_i||.
+// Eq. 2 over 32 columns: how many x_j * S/||k_j|| exceed ts = S tau ||k_i||, as two
+// partial sums.
 template <bool kMasked>
-__device__ __forceinline__ int count32(const uint32_t (&x)[32], const float* rinv,
-                                       const int* pos, int rw, uint32_t w2, float t)
+__device__ __forceinline__ float2 count32(const uint32_t (&x)[32], const float* rinv,
+                                          const int* pos, int rw, uint32_t w2, float ts)
 {
-    int c = 0;
-    const float2 mt = make_float2(-t, -t);
+    float2 ca = make_float2(0.f, 0.f), cb = make_float2(0.f, 0.f);
 #pragma unroll
     for (int k = 0; k < 32; k += 4) {
         const float4 r = *reinterpret_cast<const float4*>(rinv + k);
-        float2 a = make_float2(__uint_as_float(x[k]), __uint_as_float(x[k + 1]));
-        float2 b = make_float2(__uint_as_float(x[k + 2]), __uint_as_float(x[k + 3]));
+        float v0 = __uint_as_float(x[k]), v1 = __uint_as_float(x[k + 1]);
+        float v2 = __uint_as_float(x[k + 2]), v3 = __uint_as_float(x[k + 3]);
         if (kMasked) {
             const int4 q = *reinterpret_cast<const int4*>(pos + k);
-            a.x = (static_cast<uint32_t>(q.x - rw) > w2) ? a.x : nan_f();
-            a.y = (static_cast<uint32_t>(q.y - rw) > w2) ? a.y : nan_f();
-            b.x = (static_cast<uint32_t>(q.z - rw) > w2) ? b.x : nan_f();
-            b.y = (static_cast<uint32_t>(q.w - rw) > w2) ? b.y : nan_f();
+            v0 = (static_cast<uint32_t>(q.x - rw) > w2) ? v0 : nan_f();
+            v1 = (static_cast<uint32_t>(q.y - rw) > w2) ? v1 : nan_f();
+            v2 = (static_cast<uint32_t>(q.z - rw) > w2) ? v2 : nan_f();
+            v3 = (static_cast<uint32_t>(q.w - rw) > w2) ? v3 : nan_f();
         }
-        const float2 fa = __ffma2_rn(a, make_float2(r.x, r.y), mt);
-        const float2 fb = __ffma2_rn(b, make_float2(r.z, r.w), mt);
-        c -= static_cast<int>(gt_mask(fa.x, 0.f)) + static_cast<int>(gt_mask(fa.y, 0.f));
-        c -= static_cast<int>(gt_mask(fb.x, 0.f)) + static_cast<int>(gt_mask(fb.y, 0.f));
+        ca = __fadd2_rn(ca, make_float2(fma_sat(v0, r.x, -ts), fma_sat(v1, r.y, -ts)));
+        cb = __fadd2_rn(cb, make_float2(fma_sat(v2, r.z, -ts), fma_sat(v3, r.w, -ts)));
     }
-    return c;
+    return __fadd2_rn(ca, cb);
 }
 
 template <bool kMasked>
-__device__ __forceinline__ int count_group(const uint32_t (&x0)[32], const uint32_t (&x1)[32],
-                                           const uint32_t (&x2)[32], const uint32_t (&x3)[32],
-                                           const float* rinv, const int* pos, int rw,
-                                           uint32_t w2, float t)
+__device__ __forceinline__ float count_group(const uint32_t (&x0)[32], const uint32_t (&x1)[32],
+                                             const uint32_t (&x2)[32], const uint32_t (&x3)[32],
+                                             const float* rinv, const int* pos, int rw,
+                                             uint32_t w2, float ts)
 {
-    return count32<kMasked>(x0, rinv, pos, rw, w2, t) +
-           count32<kMasked>(x1, rinv + 32, pos + 32, rw, w2, t) +
-           count32<kMasked>(x2, rinv + 64, pos + 64, rw, w2, t) +
-           count32<kMasked>(x3, rinv + 96, pos + 96, rw, w2, t);
+    const float2 a = __fadd2_rn(count32<kMasked>(x0, rinv, pos, rw, w2, ts),
+                                count32<kMasked>(x1, rinv + 32, pos + 32, rw, w2, ts));
+    const float2 b = __fadd2_rn(count32<kMasked>(x2, rinv + 64, pos + 64, rw, w2, ts),
+                                count32<kMasked>(x3, rinv + 96, pos + 96, rw, w2, ts));
+    const float2 c = __fadd2_rn(a, b);
+    return c.x + c.y;
 }
 
 struct Tiles {
@@ -531,9 +534,12 @@ __global__ void __launch_bounds__(kThreads, 1)
 
             Best b0{-INFINITY, -1}, b1{-INFINITY, -1};   // retained (or all) / evicted
             const int rw = row - w;
-            int cnt = 0;                                   // count mode: r_i so far
-            float thr = 0.f;                               // count mode: tau * ||k_i||
-            if (kCount) thr = a.count_tau / a.colrinv[static_cast<int64_t>(u) * a.NP + row];
+            float cnt = 0.f;                               // count mode: r_i so far
+            float thr = 0.f;                               // count mode: S tau ||k_i||
+            if (kCount)
+                thr = (a.count_tau /
+                       (a.colrinv[static_cast<int64_t>(u) * a.NP + row] * (1.0f / kCountScale))) *
+                      kCountScale;
             for (int t = 0; t < nt; ++t) {
                 ok = all_wait(&m_full[ms], mph, wc, 7);
                 if (ok) ok = all_wait(&t_full[acc], tph, wc, 8);
@@ -591,18 +597,18 @@ __global__ void __launch_bounds__(kThreads, 1)
                 ok = all_wait(&x_empty[xb], ((n_x >> 1) & 1) ^ 1, wc, 9);
                 if (!ok) break;
                 X[(h - 1) * kBM + row_local] =
-                    kCount ? make_float4(__int_as_float(cnt), 0.f, 0.f, 0.f)
+                    kCount ? make_float4(cnt, 0.f, 0.f, 0.f)
                            : make_float4(bv0, __int_as_float(bc0), bv1, __int_as_float(bc1));
                 mbar_arrive(&x_full[xb]);
             } else if (kCount) {
                 ok = all_wait(&x_full[xb], (n_x >> 1) & 1, wc, 10);
                 if (!ok) break;
-                int total = cnt;
+                float total = cnt;
 #pragma unroll
-                for (int g = 1; g < kGroups; ++g)
-                    total += __float_as_int(X[(g - 1) * kBM + row_local].x);
+                for (int g = 1; g < kGroups; ++g) total += X[(g - 1) * kBM + row_local].x;
                 mbar_arrive(&x_empty[xb]);
-                if (row < a.N) a.out_count[static_cast<int64_t>(u) * a.N + row] = total;
+                if (row < a.N)
+                    a.out_count[static_cast<int64_t>(u) * a.N + row] = __float2int_rn(total);
             } else {
                 ok = all_wait(&x_full[xb], (n_x >> 1) & 1, wc, 10);
                 if (!ok) break;

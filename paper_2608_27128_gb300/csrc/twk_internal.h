@@ -33,7 +33,8 @@ struct AuditArgs {
     uint32_t mant_mask;         // 0xFFFFFFE0: clears the 5 mantissa bits that carry the
                                 // column; a runtime value, so the compiler keeps it in a
                                 // register and the pack is a single 3-input logic op
-    // count mode (Eq. 2): mode 0 columns only; out_t0/out_t1 unused
+    // count mode (Eq. 2): mode 0 columns only, colrinv scaled by kCountScale;
+    // out_t0/out_t1 unused
     float count_tau;            // tau, compared strictly
     int* out_count;             // [U][N] r_i
 };
@@ -58,14 +59,20 @@ struct RepairArgs {
     int* rank_of;               // [U][N] scratch: donor rank of each position
 };
 
+// The count mode's column scales are 1/||k|| times this power of two: one saturated
+// fused multiply-add per pair then gives exactly 1 or 0 (see twk_audit.cu).
+constexpr float kCountScale = 0x1p32f;
+
 // Largest N the dedup variant accepts: its walk keeps 2 bits per donor in shared memory.
 constexpr int kDedupMaxN = 1 << 19;
 
 // prep kernels
 cudaError_t launch_round_bf16(const float* in, uint16_t* out, int64_t n, cudaStream_t st);
 // NP must be a multiple of 64 (column_stride gives a multiple of 256).
+// rscale: a power of two that multiplies every colrinv (1 except for the count mode)
 cudaError_t launch_norms_identity(const uint16_t* keys, int U, int N, int d, int64_t NP,
-                                  float* colrinv, int* colpos, float4* norms, cudaStream_t st);
+                                  float* colrinv, int* colpos, float4* norms, cudaStream_t st,
+                                  float rscale = 1.0f);
 cudaError_t launch_scan(const uint8_t* mask, int U, int N, int* cnt, int* kb, cudaStream_t st);
 cudaError_t launch_gather(const uint16_t* keys, const uint8_t* mask, const int* cnt,
                           const int* kb, int U, int N, int d, int64_t NP, uint16_t* kp,

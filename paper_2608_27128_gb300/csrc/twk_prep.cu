@@ -39,14 +39,15 @@ __device__ __forceinline__ float4 key_norms(const uint16_t* key, int part, float
     return make_float4(sq.h, sq.l, rn.h, rn.l);
 }
 
-// Mode 0 (keys as given): per column p of unit blockIdx.y, colrinv = 1/||k_p|| and
-// colpos = p, NaN / -1 on the padding columns [N, NP); norms[u][p] = the norm record.
+// Mode 0 (keys as given): per column p of unit blockIdx.y, colrinv = rscale/||k_p||
+// (rscale a power of two, so the scaling is exact) and colpos = p, NaN / -1 on the
+// padding columns [N, NP); norms[u][p] = the norm record.
 // Grid (NP / kKeysPerBlock, U), kParts lanes per column.
 template <int D>
 __global__ void __launch_bounds__(kPrepThreads)
     norms_identity_kernel(const uint16_t* __restrict__ keys, int N, int64_t NP,
                           float* __restrict__ colrinv, int* __restrict__ colpos,
-                          float4* __restrict__ norms)
+                          float4* __restrict__ norms, float rscale)
 {
     const int part = threadIdx.x % kParts;
     const int p = blockIdx.x * kKeysPerBlock + threadIdx.x / kParts;
@@ -56,7 +57,7 @@ __global__ void __launch_bounds__(kPrepThreads)
     float r32;
     const float4 nr = key_norms<D>(keys + (u * N + pk) * D, part, r32);
     if (part == 0) {
-        colrinv[u * NP + p] = p < N ? r32 : nan_f();
+        colrinv[u * NP + p] = p < N ? r32 * rscale : nan_f();
         colpos[u * NP + p] = p < N ? p : -1;
         if (p < N) norms[u * N + p] = nr;
     }
@@ -159,13 +160,16 @@ cudaError_t launch_round_bf16(const float* in, uint16_t* out, int64_t n, cudaStr
 }
 
 cudaError_t launch_norms_identity(const uint16_t* keys, int U, int N, int d, int64_t NP,
-                                  float* colrinv, int* colpos, float4* norms, cudaStream_t st)
+                                  float* colrinv, int* colpos, float4* norms, cudaStream_t st,
+                                  float rscale)
 {
     const dim3 grid(static_cast<unsigned>(NP / kKeysPerBlock), U);
     if (d == 128)
-        norms_identity_kernel<128><<<grid, kPrepThreads, 0, st>>>(keys, N, NP, colrinv, colpos, norms);
+        norms_identity_kernel<128><<<grid, kPrepThreads, 0, st>>>(keys, N, NP, colrinv, colpos,
+                                                                   norms, rscale);
     else
-        norms_identity_kernel<64><<<grid, kPrepThreads, 0, st>>>(keys, N, NP, colrinv, colpos, norms);
+        norms_identity_kernel<64><<<grid, kPrepThreads, 0, st>>>(keys, N, NP, colrinv, colpos,
+                                                                  norms, rscale);
     return cudaGetLastError();
 }
 
