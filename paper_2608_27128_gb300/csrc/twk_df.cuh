@@ -83,6 +83,75 @@ __device__ __forceinline__ DFPair group_dot_df(const uint16_t* __restrict__ a,
     return DFPair{hi, lo};
 }
 
+// The same two dot products a . b0 and a . b1 at once, one in each half of paired
+// (f32x2) instructions: each half performs exactly the scalar sequence of
+// group_dot_df, with the same rounding, term order and combine tree, so each result
+// equals group_dot_df's bit for bit.
+__device__ __forceinline__ float2 neg2(float2 a) { return make_float2(-a.x, -a.y); }
+
+__device__ __forceinline__ void two_sum_acc2(float2& hi, float2& lo, float2 p)
+{
+    const float2 s = __fadd2_rn(hi, p);
+    const float2 bp = __fadd2_rn(s, neg2(hi));
+    const float2 e = __fadd2_rn(__fadd2_rn(hi, neg2(__fadd2_rn(s, neg2(bp)))),
+                                __fadd2_rn(p, neg2(bp)));
+    hi = s;
+    lo = __fadd2_rn(lo, e);
+}
+
+__device__ __forceinline__ void df_add2(float2& hi, float2& lo, float2 hi2, float2 lo2)
+{
+    const float2 s = __fadd2_rn(hi, hi2);
+    const float2 bp = __fadd2_rn(s, neg2(hi));
+    float2 e = __fadd2_rn(__fadd2_rn(hi, neg2(__fadd2_rn(s, neg2(bp)))), __fadd2_rn(hi2, neg2(bp)));
+    e = __fadd2_rn(e, __fadd2_rn(lo, lo2));
+    hi = __fadd2_rn(s, e);
+    lo = __fadd2_rn(e, neg2(__fadd2_rn(hi, neg2(s))));
+}
+
+template <int D>
+__device__ __forceinline__ void group_dot2_df(const uint16_t* __restrict__ a,
+                                              const uint16_t* __restrict__ b0,
+                                              const uint16_t* __restrict__ b1, int part,
+                                              DFPair& r0, DFPair& r1)
+{
+    constexpr int Q = D / 8 / kParts;
+    const uint4* a4 = reinterpret_cast<const uint4*>(a) + part * Q;
+    const uint4* c4 = reinterpret_cast<const uint4*>(b0) + part * Q;
+    const uint4* d4 = reinterpret_cast<const uint4*>(b1) + part * Q;
+    float2 hi = make_float2(0.f, 0.f), lo = make_float2(0.f, 0.f);
+#pragma unroll
+    for (int q = 0; q < Q; ++q) {
+        const uint4 va = __ldg(a4 + q);
+        const uint4 vc = __ldg(c4 + q);
+        const uint4 vd = __ldg(d4 + q);
+        const uint32_t wa[4] = {va.x, va.y, va.z, va.w};
+        const uint32_t wc[4] = {vc.x, vc.y, vc.z, vc.w};
+        const uint32_t wd[4] = {vd.x, vd.y, vd.z, vd.w};
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            const float lo_a = __uint_as_float(wa[k] << 16);
+            const float hi_a = __uint_as_float(wa[k] & 0xFFFF0000u);
+            two_sum_acc2(hi, lo, __fmul2_rn(make_float2(lo_a, lo_a),
+                                            make_float2(__uint_as_float(wc[k] << 16),
+                                                        __uint_as_float(wd[k] << 16))));
+            two_sum_acc2(hi, lo, __fmul2_rn(make_float2(hi_a, hi_a),
+                                            make_float2(__uint_as_float(wc[k] & 0xFFFF0000u),
+                                                        __uint_as_float(wd[k] & 0xFFFF0000u))));
+        }
+    }
+#pragma unroll
+    for (int o = 1; o < kParts; o <<= 1) {
+        const float2 h2 = make_float2(__shfl_xor_sync(0xFFFFFFFFu, hi.x, o),
+                                      __shfl_xor_sync(0xFFFFFFFFu, hi.y, o));
+        const float2 l2 = make_float2(__shfl_xor_sync(0xFFFFFFFFu, lo.x, o),
+                                      __shfl_xor_sync(0xFFFFFFFFu, lo.y, o));
+        df_add2(hi, lo, h2, l2);
+    }
+    r0 = DFPair{hi.x, lo.x};
+    r1 = DFPair{hi.y, lo.y};
+}
+
 // ---- double-float (unevaluated fp32 pair) helpers --------------------------------
 
 using DF = DFPair;

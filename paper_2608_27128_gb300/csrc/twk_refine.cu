@@ -12,9 +12,10 @@
 // cosine is then (k_i . k_j) * (1/||k_i|| * 1/||k_j||) in double-float arithmetic
 // (relative error below 1e-12; fp64 square roots and quotients are slow on this GPU),
 // except within 2^-20 of +-1, where the exact fp64 form is used.  All dot products
-// (norms included) use the same routine and term order, and the product of the two
-// inverse norms is formed symmetrically, so the result is symmetric in (i, j) bit for
-// bit and exactly 1 for a duplicate.
+// (norms included) use the same routine and term order (the paired version used when a
+// row has two candidates computes each dot exactly as the single one), and the product
+// of the two inverse norms is formed symmetrically, so the result is symmetric in
+// (i, j) bit for bit and exactly 1 for a duplicate.
 #include "twk_df.cuh"
 #include "twk_internal.h"
 
@@ -60,13 +61,12 @@ __global__ void __launch_bounds__(kRefineThreads)
     // Every lane of the warp takes part in the shuffled dot products; a missing twin is
     // stood in for by the row itself and its value discarded.
     const int64_t s0 = base + (j0 >= 0 ? j0 : r - base);
-    const DF d0 = group_dot_df<D>(ki, keys + s0 * D, part);
-    DF d1{0.f, 0.f};
-    int64_t s1 = s0;
-    if (__any_sync(0xFFFFFFFFu, j1 >= 0)) {
-        s1 = base + (j1 >= 0 ? j1 : r - base);
-        d1 = group_dot_df<D>(ki, keys + s1 * D, part);
-    }
+    const int64_t s1 = base + (j1 >= 0 ? j1 : r - base);
+    DF d0, d1{0.f, 0.f};
+    if (__any_sync(0xFFFFFFFFu, j1 >= 0))   // both dots at once, one per f32x2 half
+        group_dot2_df<D>(ki, keys + s0 * D, keys + s1 * D, part, d0, d1);
+    else
+        d0 = group_dot_df<D>(ki, keys + s0 * D, part);
     // lane 0 of the group evaluates the first cosine, lane 1 the second
     double v = -1.0;
     if (part == 0 && j0 >= 0) v = cosine(d0, norms[r], norms[s0]);
