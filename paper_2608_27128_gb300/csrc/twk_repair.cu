@@ -86,6 +86,75 @@ __device__ __forceinline__ void scan2(Shared& s, int fo, int fd, int& po, int& p
     __syncthreads();
 }
 
+// Called by warp 0 only: the 256 digit counts in cnt become their exclusive prefix
+// (eight digits per lane and a shuffle scan); returns whether one digit holds all n.
+__device__ __forceinline__ bool digit_prefix(int* cnt, int n)
+{
+    const int lane = threadIdx.x & 31;
+    int c[8], t = 0;
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+        c[j] = cnt[lane * 8 + j];
+        t += c[j];
+    }
+    int incl = t;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xFFFFFFFFu, incl, o);
+        if (lane >= o) incl += y;
+    }
+    int run = incl - t;
+    bool one = false;
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+        one |= c[j] == n;
+        cnt[lane * 8 + j] = run;
+        run += c[j];
+    }
+    return __any_sync(0xFFFFFFFFu, one);
+}
+
+// Called by warp 0 only: the smallest digit d whose counts up to and including d reach
+// `need` (255 at most), the count before it and its own count, into s.
+__device__ __forceinline__ void digit_cut(const int* cnt, int need, int& sel_digit,
+                                          int& sel_before, int& sel_count)
+{
+    const int lane = threadIdx.x & 31;
+    int c[8], t = 0;
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+        c[j] = cnt[lane * 8 + j];
+        t += c[j];
+    }
+    int incl = t;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xFFFFFFFFu, incl, o);
+        if (lane >= o) incl += y;
+    }
+    const uint32_t reach = __ballot_sync(0xFFFFFFFFu, incl >= need);
+    const int L = reach ? __ffs(reach) - 1 : 31;
+    if (lane == L) {
+        // the first of the lane's digits whose running count reaches need (its last
+        // digit otherwise: digit 255 for lane 31); constant indices keep c in registers
+        int run = incl - t, sel = 7, before = 0, count = c[7];
+        bool found = false;
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+            if (!found && (j == 7 || run + c[j] >= need)) {
+                sel = j;
+                before = run;
+                count = c[j];
+                found = true;
+            }
+            if (!found) run += c[j];
+        }
+        sel_digit = L * 8 + sel;
+        sel_before = before;
+        sel_count = count;
+    }
+}
+
 // One stable counting pass on digit (key >> shift) & 255 of n items; returns false
 // (and moves nothing) when every item has the same digit.
 __device__ bool radix_pass(Shared& s, const uint64_t* kin, const int* iin, uint64_t* kout,
@@ -102,15 +171,9 @@ __device__ bool radix_pass(Shared& s, const uint64_t* kin, const int* iin, uint6
         if (dg < 256 && lane == __ffs(peers) - 1) atomicAdd(&s.base[dg], __popc(peers));
     }
     __syncthreads();
-    if (threadIdx.x == 0) {
-        int run = 0, single = 0;
-        for (int d = 0; d < 256; ++d) {
-            const int c = s.base[d];
-            if (c == n) single = 1;
-            s.base[d] = run;
-            run += c;
-        }
-        s.flag = single;
+    if (threadIdx.x < 32) {
+        const bool single = digit_prefix(s.base, n);
+        if (threadIdx.x == 0) s.flag = single;
     }
     __syncthreads();
     if (s.flag) return false;
@@ -188,13 +251,7 @@ __device__ void select_smallest(Shared& s, const uint64_t* kin, const int* iin, 
             if (dg < 256 && lane == __ffs(peers) - 1) atomicAdd(&s.base[dg], __popc(peers));
         }
         __syncthreads();
-        if (threadIdx.x == 0) {
-            int run = 0, d = 0;
-            for (; d < 255 && run + s.base[d] < need; ++d) run += s.base[d];
-            s.sel_digit = d;
-            s.sel_before = run;
-            s.sel_count = s.base[d];
-        }
+        if (threadIdx.x < 32) digit_cut(s.base, need, s.sel_digit, s.sel_before, s.sel_count);
         __syncthreads();
         need -= s.sel_before;
         prefix |= static_cast<uint64_t>(s.sel_digit) << shift;
@@ -252,7 +309,7 @@ inline size_t dedup_smem_bytes(int N)
 }
 
 template <bool kDedup>
-__global__ void __launch_bounds__(kT, 1) repair_kernel(const RepairArgs a)
+__global__ void __launch_bounds__(kT, 2) repair_kernel(const RepairArgs a)   // 2 blocks/SM
 {
     __shared__ Shared s;
     const int u = blockIdx.x;
