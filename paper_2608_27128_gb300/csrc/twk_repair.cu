@@ -155,6 +155,53 @@ __device__ __forceinline__ void digit_cut(const int* cnt, int need, int& sel_dig
     }
 }
 
+// Block-wide exclusive scan of two per-thread counts; returns each thread's prefixes
+// and the totals.
+__device__ __forceinline__ void scan2n(Shared& s, int co, int cd, int& po, int& pd, int& to,
+                                       int& td)
+{
+    const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+    int io = co, id = cd;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const int yo = __shfl_up_sync(0xFFFFFFFFu, io, o);
+        const int yd = __shfl_up_sync(0xFFFFFFFFu, id, o);
+        if (lane >= o) {
+            io += yo;
+            id += yd;
+        }
+    }
+    if (lane == 31) {
+        s.wsum[0][wid] = io;
+        s.wsum[1][wid] = id;
+    }
+    __syncthreads();
+    if (wid == 0) {
+        int x = lane < kW ? s.wsum[0][lane] : 0, y = lane < kW ? s.wsum[1][lane] : 0;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int xo = __shfl_up_sync(0xFFFFFFFFu, x, o);
+            const int yo = __shfl_up_sync(0xFFFFFFFFu, y, o);
+            if (lane >= o) {
+                x += xo;
+                y += yo;
+            }
+        }
+        if (lane < kW) {
+            s.wsum[0][lane] = x;   // inclusive
+            s.wsum[1][lane] = y;
+        }
+    }
+    __syncthreads();
+    po = (wid ? s.wsum[0][wid - 1] : 0) + io - co;
+    pd = (wid ? s.wsum[1][wid - 1] : 0) + id - cd;
+    to = s.wsum[0][kW - 1];
+    td = s.wsum[1][kW - 1];
+    __syncthreads();
+}
+
+constexpr int kE = 4;   // consecutive positions per thread in the streaming passes
+
 // One stable counting pass on digit (key >> shift) & 255 of n items; returns false
 // (and moves nothing) when every item has the same digit.
 __device__ bool radix_pass(Shared& s, const uint64_t* kin, const int* iin, uint64_t* kout,
@@ -320,16 +367,24 @@ __global__ void __launch_bounds__(kT, 2) repair_kernel(const RepairArgs a)   // 
     uint8_t* S1 = a.out_mask + off;
     int* swaps = a.out_swaps + static_cast<int64_t>(u) * 2 * (N / 2);
 
-    // 1. validation
+    // 1. validation, counts, and S1 = S0 (also the answer for a failed unit or m = 0)
     int bad = 0, cnt = 0, no = 0, nd = 0;
     const double tau = a.tau;
-    for (int i = threadIdx.x; i < N; i += kT) {
-        const uint8_t v = S0[i];
-        bad |= v > 1;
-        cnt += v != 0;
-        const bool prot = i < a.n_sink || i >= N - a.n_recent;
-        no += (v == 0 && b[i] < tau);
-        nd += (v != 0 && !prot && b[i] >= tau);
+    for (int c0 = 0; c0 < N; c0 += kT * kE) {
+#pragma unroll
+        for (int j = 0; j < kE; ++j) {
+            const int i = c0 + threadIdx.x * kE + j;
+            if (i < N) {
+                const uint8_t v = S0[i];
+                const double bi = b[i];
+                S1[i] = v;
+                bad |= v > 1;
+                cnt += v != 0;
+                const bool prot = i < a.n_sink || i >= N - a.n_recent;
+                no += (v == 0 && bi < tau);
+                nd += (v != 0 && !prot && bi >= tau);
+            }
+        }
     }
     if (threadIdx.x < 4) s.red[threadIdx.x] = 0;
     __syncthreads();
@@ -350,8 +405,6 @@ __global__ void __launch_bounds__(kT, 2) repair_kernel(const RepairArgs a)   // 
     const int n_o = s.red[2], n_d = s.red[3];
     const int m = status ? 0 : min(n_o, n_d);
 
-    // S1 starts as S0 (also the answer for a failed unit or m = 0).
-    for (int i = threadIdx.x; i < N; i += kT) S1[i] = S0[i];
     if (status != 0 || m == 0) {
         if (threadIdx.x == 0) {
             a.out_nswaps[u] = status ? -1 : 0;
@@ -366,26 +419,39 @@ __global__ void __launch_bounds__(kT, 2) repair_kernel(const RepairArgs a)   // 
     uint64_t* k1 = a.keys1 + off;
     int* i1 = a.idx1 + off;
     int base_o = 0, base_d = n_o;
-    for (int c0 = 0; c0 < N; c0 += kT) {
-        const int i = c0 + threadIdx.x;
-        int fo = 0, fd = 0;
-        double bi = 0.0;
-        if (i < N) {
-            const uint8_t v = S0[i];
-            bi = b[i];
-            const bool prot = i < a.n_sink || i >= N - a.n_recent;
-            fo = (v == 0 && bi < tau);
-            fd = (v != 0 && !prot && bi >= tau);
+    for (int c0 = 0; c0 < N; c0 += kT * kE) {
+        int fo[kE], fd[kE], co = 0, cd = 0;
+        double bv[kE];
+#pragma unroll
+        for (int j = 0; j < kE; ++j) {
+            const int i = c0 + threadIdx.x * kE + j;
+            fo[j] = fd[j] = 0;
+            bv[j] = 0.0;
+            if (i < N) {
+                const uint8_t v = S0[i];
+                bv[j] = b[i];
+                const bool prot = i < a.n_sink || i >= N - a.n_recent;
+                fo[j] = (v == 0 && bv[j] < tau);
+                fd[j] = (v != 0 && !prot && bv[j] >= tau);
+            }
+            co += fo[j];
+            cd += fd[j];
         }
         int po, pd, to, td;
-        scan2(s, fo, fd, po, pd, to, td);
-        if (fo) {
-            k0[base_o + po] = ordered(bi);
-            i0[base_o + po] = i;
-        }
-        if (fd) {
-            k0[base_d + pd] = ~ordered(bi);
-            i0[base_d + pd] = i;
+        scan2n(s, co, cd, po, pd, to, td);
+#pragma unroll
+        for (int j = 0; j < kE; ++j) {
+            const int i = c0 + threadIdx.x * kE + j;
+            if (fo[j]) {
+                k0[base_o + po] = ordered(bv[j]);
+                i0[base_o + po] = i;
+                ++po;
+            }
+            if (fd[j]) {
+                k0[base_d + pd] = ~ordered(bv[j]);
+                i0[base_d + pd] = i;
+                ++pd;
+            }
         }
         base_o += to;
         base_d += td;
