@@ -45,18 +45,24 @@ def peaks():
         return dict(FALLBACK), "fallback"
 
 
+WORKLOAD_NAMES = {"qwen": "Qwen3-4B KV cache", "llama": "Llama-3.2-1B KV cache",
+                  "retrieval": "Qwen3-4B retrieval-style cache",
+                  "long": "long single-layer stress cache"}
+
+
 def workload_config(w, ratio, path="repair"):
     what = {"repair": "audit + repair (Sec. 3.4)",
             "dedup": "audit + repair that keeps one member of each twin pair (Sec. 3.4)",
             "policy": "standalone policy: counts + selection (Sec. 3.2 Eq. 2-3)"}[path]
+    kbytes = w.L * w.H * w.N * w.d * 2
     return {
-        "workload": f"Qwen3-4B KV cache {w.L}x{w.H}x{w.N}x{w.d} bf16 (synthetic), ratio {ratio}, "
-                    f"{what}",
+        "workload": f"{WORKLOAD_NAMES[w.name]} {w.L}x{w.H}x{w.N}x{w.d} bf16 (synthetic), "
+                    f"ratio {ratio}, {what}",
         "path": path,
         "L": w.L, "H": w.H, "N": w.N, "d": w.d, "ratio": ratio, "tau": w.tau,
         "window": 32, "n_sink": 4, "n_recent": 64,
         "budget_per_unit": None,
-        "l2": "inputs larger than L2 (keys 1.2 GB > 129 MB); no flush",
+        "l2": f"inputs larger than L2 (keys {kbytes / 1e9:.2f} GB > 129 MB); no flush",
         "parallelism": "replicas",
     }
 
@@ -162,6 +168,7 @@ def cpu_sample(w, ratio, units, rows_per_unit, path="repair"):
     ul = [(u // w.H, u % w.H) for u in range(units)]
     keys, _ = synth.keys(w, units=ul)
     S0 = synth.masks(w, ratio, units=ul)
+    rows_per_unit = max(256, min(w.N, rows_per_unit * 16384 // w.N))   # same work per row set
     rows = np.sort(np.random.default_rng(0).choice(w.N, size=rows_per_unit, replace=False))
     t0 = time.perf_counter()
     if path == "policy":
@@ -272,7 +279,8 @@ def run_ours(args, w, ratio):
 
     if rank != 0:
         return
-    _report(args, w, ratio, world, U, N, d, ms, prof, e2e_ms, h2d, d2h, chunk, clocks)
+    m_total = int(out["nswaps"].clamp(min=0).sum().item()) if "nswaps" in out else 0
+    _report(args, w, ratio, world, U, N, d, ms, prof, e2e_ms, h2d, d2h, chunk, clocks, m_total)
 
 
 def run_e2e(args, world, w, keys_h, mask_h, budget_h, out, stream):
@@ -326,7 +334,38 @@ def run_e2e(args, world, w, keys_h, mask_h, budget_h, out, stream):
     return e2e_ms, h2d, d2h, chunk
 
 
-def _report(args, w, ratio, world, U, N, d, ms, prof, e2e_ms, h2d, d2h, chunk, clocks):
+def kernel_bytes(path, U, N, d, m_total):
+    """Algorithmic DRAM bytes per step of the memory-bound kernels (the per-unit
+    figures of the design notes times the units; swaps counted as 8 bytes each)."""
+    NP = ((N + 255) // 256) * 256 + 256
+    if path == "policy":
+        return {"prep": U * (N * d * 2 + 8 * NP + 16 * N),          # norms, identity layout
+                "repair": U * (4 * N + N)}                             # counts in, mask out
+    return {"prep": U * (5 * N + N + N * d * 2 + NP * d * 2 + 8 * NP + 16 * N),   # scan + gather
+            "repair": U * (8 * N + N + N) + 8 * m_total,               # b, S0 in; S1 out; swaps
+            "refine": U * N * (2 * d + 40)}                            # k_i, norms, twins, scores
+
+
+def cpu_sample_1thread(w, ratio, path, rows=1024):
+    """The oracle on one host core (OMP_NUM_THREADS=1 in a child process): 1 unit x `rows`
+    rows, every column.  Returns the cpu_baseline-style record, or None."""
+    code = ("import json,sys; sys.path.insert(0, %r); import bench; "
+            "from paper_2608_27128_gb300 import synth; "
+            "w = synth.get(%r, L=%d); v, dt, t, desc = bench.cpu_sample(w, %r, 1, %d, %r); "
+            "print(json.dumps([v, dt, t, desc]))") % (ROOT, w.name, w.L, ratio, rows, path)
+    env = dict(os.environ, OMP_NUM_THREADS="1")
+    try:
+        p = subprocess.run([sys.executable, "-c", code], capture_output=True, text=True,
+                           env=env, timeout=300)
+        v, dt, t, desc = json.loads(p.stdout.strip().splitlines()[-1])
+        return {"value": v, "unit": "keys/s", "cores": t, "kind": "oracle", "sample": desc,
+                "seconds": dt}
+    except (subprocess.SubprocessError, ValueError, IndexError):
+        return None
+
+
+def _report(args, w, ratio, world, U, N, d, ms, prof, e2e_ms, h2d, d2h, chunk, clocks,
+            m_total=0):
     value = job_throughput(world, U * N, ms)
     # ---- roofline of the dominant kernel (the fused audit)
     pk, pk_kind = peaks()
@@ -363,10 +402,25 @@ def _report(args, w, ratio, world, U, N, d, ms, prof, e2e_ms, h2d, d2h, chunk, c
             **getattr(args, "e2e_step_stats", {})},
         "clocks": clocks.summary(),
     }
+    # memory-bound kernels against the measured copy bandwidth
+    kb = kernel_bytes(args.path, U, N, d, m_total)
+    line["kernels"] = {}
+    for k, (n, t) in prof.items():
+        if t <= 0:
+            continue
+        rec = {"ms_per_step": t / args.steps}
+        if k in kb:
+            gbs = kb[k] / (t / args.steps * 1e-3) / 1e9
+            rec.update({"algorithmic_bytes": kb[k], "gbs": gbs,
+                        "frac_of_hbm": gbs / pk["hbm_gbs"]})
+        line["kernels"][k] = rec
     if not args.no_cpu:
         v, dt, threads, desc = cpu_sample(w, ratio, args.cpu_units, args.cpu_rows, args.path)
         line["cpu_baseline"] = {"value": v, "unit": "keys/s", "cores": threads,
                                 "kind": "oracle", "sample": desc, "seconds": dt}
+        one = cpu_sample_1thread(w, ratio, args.path)
+        if one is not None:
+            line["cpu_baseline_1core"] = one
     print(json.dumps(line), flush=True)
 
 
@@ -415,11 +469,16 @@ def main():
                     help="repair: audit + swap (the headline); dedup: the repair that "
                          "never evicts both members of a twin pair; policy: the "
                          "standalone scorer of Sec. 3.2")
+    ap.add_argument("--workload", choices=("qwen", "llama", "retrieval", "long"),
+                    default="qwen",
+                    help="qwen: the Qwen3-4B cache shape the metric is quoted on (the "
+                         "default line); the others are reported alongside")
     ap.add_argument("--layers", type=int, default=None,
                     help="fewer layers of the same workload (for profiler captures)")
     args = ap.parse_args()
     from paper_2608_27128_gb300 import synth
-    w = synth.get("qwen") if args.layers is None else synth.get("qwen", L=args.layers)
+    w = synth.get(args.workload) if args.layers is None else synth.get(args.workload,
+                                                                        L=args.layers)
     if args.impl == "reference":
         run_reference(args, w, args.ratio)
     else:
