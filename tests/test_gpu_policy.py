@@ -3,7 +3,7 @@ with the fp64 oracle.
 
 - Counts: each row's r_i must lie in [r(tau + BAND), r(tau - BAND)] of the oracle, so
   it equals the oracle's count wherever no pair's similarity lies within BAND of tau.
-  BAND = 1e-4 is far below the spec tie band (4e-3) and far above the fp32
+  BAND = 1e-4 is far below the score tie band of 4e-3 and far above the fp32
   error of the kernel's decision (about 1e-6).
 - Selection: the oracle's selection fed the GPU's own counts reproduces the mask and
   statuses bit for bit (split check).
