@@ -50,18 +50,22 @@ WORKLOAD_NAMES = {"qwen": "Qwen3-4B KV cache", "llama": "Llama-3.2-1B KV cache",
                   "long": "long single-layer stress cache"}
 
 
-def workload_config(w, ratio, path="repair"):
+def workload_config(w, ratio, path="repair", schedule="uniform"):
+    from paper_2608_27128_gb300 import synth
     what = {"repair": "audit + repair (Sec. 3.4)",
             "dedup": "audit + repair that keeps one member of each twin pair (Sec. 3.4)",
             "policy": "standalone policy: counts + selection (Sec. 3.2 Eq. 2-3)"}[path]
     kbytes = w.L * w.H * w.N * w.d * 2
+    per_layer = (synth.pyramid_budgets(w, ratio).tolist() if schedule == "pyramid" else None)
     return {
         "workload": f"{WORKLOAD_NAMES[w.name]} {w.L}x{w.H}x{w.N}x{w.d} bf16 (synthetic), "
-                    f"ratio {ratio}, {what}",
+                    f"ratio {ratio}" + (", per-layer pyramid budgets" if per_layer else "") +
+                    f", {what}",
         "path": path,
         "L": w.L, "H": w.H, "N": w.N, "d": w.d, "ratio": ratio, "tau": w.tau,
         "window": 32, "n_sink": 4, "n_recent": 64,
-        "budget_per_unit": None,
+        "schedule": schedule,
+        "budget_per_layer": per_layer,
         "l2": f"inputs larger than L2 (keys {kbytes / 1e9:.2f} GB > 129 MB); no flush",
         "parallelism": "replicas",
     }
@@ -202,7 +206,7 @@ def run_reference(args, w, ratio):
         "metric": METRIC, "value": v, "unit": "keys/s", "n_gpus": args.gpus,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
-        "data": "synthetic", "config": workload_config(w, ratio, args.path), "impl": "reference",
+        "data": "synthetic", "config": workload_config(w, ratio, args.path, args.schedule), "impl": "reference",
         "cpu_baseline": {"value": v, "unit": "keys/s", "cores": threads, "kind": "oracle",
                          "sample": desc},
         "e2e": {"value": v, "unit": "keys/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
@@ -222,7 +226,7 @@ def run_ours(args, w, ratio):
     tk.load()
 
     keys_np, _ = synth.keys(w)
-    S0_np = synth.masks(w, ratio)
+    S0_np = synth.masks(w, ratio, schedule=args.schedule)
     L, H, N, d = w.L, w.H, w.N, w.d
     U = L * H
     keys_h = torch.from_numpy(keys_np.view(np.int16).reshape(L, H, N, d)).view(torch.bfloat16)
@@ -237,7 +241,10 @@ def run_ours(args, w, ratio):
 
     if args.path == "policy":
         ws = tk.workspace(shape, tk.OP_POLICY, dev)
-        K = torch.full((U,), tk.budget_for_ratio(N, ratio), dtype=torch.int32, device=dev)
+        if args.schedule == "pyramid":
+            K = torch.from_numpy(np.repeat(synth.pyramid_budgets(w, ratio), H).astype(np.int32)).to(dev)
+        else:
+            K = torch.full((U,), tk.budget_for_ratio(N, ratio), dtype=torch.int32, device=dev)
 
     def step(k=keys, m=mask, b=budget):
         nonlocal out
@@ -381,7 +388,7 @@ def _report(args, w, ratio, world, U, N, d, ms, prof, e2e_ms, h2d, d2h, chunk, c
         "metric": METRIC, "value": value, "unit": "keys/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
-        "data": "synthetic", "config": workload_config(w, ratio, args.path),
+        "data": "synthetic", "config": workload_config(w, ratio, args.path, args.schedule),
         "tflops_audit": achieved,
         "frac_of_burst_peak": achieved / pk["bf16_tflops"],
         "roofline": {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
@@ -473,6 +480,9 @@ def main():
                     default="qwen",
                     help="qwen: the Qwen3-4B cache shape the metric is quoted on (the "
                          "default line); the others are reported alongside")
+    ap.add_argument("--schedule", choices=("uniform", "pyramid"), default="uniform",
+                    help="uniform: one budget for every unit (the default line); pyramid: "
+                         "per-layer budgets shrinking with depth, same total")
     ap.add_argument("--layers", type=int, default=None,
                     help="fewer layers of the same workload (for profiler captures)")
     args = ap.parse_args()

@@ -220,6 +220,29 @@ def budget(w: Workload, ratio: float) -> int:
     return int(math.ceil((1.0 - ratio) * w.N - 1e-9))
 
 
+def pyramid_budgets(w: Workload, ratio: float, spread: float = 0.5) -> np.ndarray:
+    """Per-layer retained counts that shrink linearly with depth, as layer-wise budget
+    schedules do (the policies the repair wraps may give each layer its own budget,
+    Sec. 4.1): layer l gets about mean * (1 + s * (1 - 2 l / (L - 1))), i.e.
+    (1 + s) * mean at the first layer and (1 - s) * mean at the last, with s = spread
+    reduced where needed so that both ends stay within [n_sink + n_recent, N].  The
+    counts are integers summing to exactly L * mean: the floors, plus one for the
+    layers with the largest fractional parts (lower layer first on ties).  Every head
+    of a layer shares the layer's count.  Returns int64 [L]."""
+    mean = budget(w, ratio)
+    L, N = w.L, w.N
+    if L == 1:
+        return np.array([mean], np.int64)
+    lo = min(N_SINK + N_RECENT, N)
+    s = max(0.0, min(spread, (N - mean) / mean, (mean - lo) / mean))
+    raw = np.array([mean * (1.0 + s * (1.0 - 2.0 * l / (L - 1))) for l in range(L)])
+    k = np.floor(raw).astype(np.int64)
+    rest = int(L * mean - k.sum())          # 0 <= rest < L: the schedule sums to L * mean
+    order = np.argsort(-(raw - k), kind="stable")
+    k[order[:rest]] += 1
+    return np.clip(k, lo, N)
+
+
 def _top_k(scores: np.ndarray, forced: np.ndarray, K: int) -> np.ndarray:
     """Retain every forced position, then the highest scores (lower index on ties)."""
     N = scores.size
@@ -233,10 +256,11 @@ def _top_k(scores: np.ndarray, forced: np.ndarray, K: int) -> np.ndarray:
     return mask
 
 
-def unit_mask(w: Workload, layer: int, head: int, ratio: float) -> np.ndarray:
-    """Retained set S0 of one unit from the workload's stand-in policy."""
+def unit_mask(w: Workload, layer: int, head: int, ratio: float, K: int | None = None) -> np.ndarray:
+    """Retained set S0 of one unit from the workload's stand-in policy (K retained;
+    default the workload's uniform budget for `ratio`)."""
     N = w.N
-    K = budget(w, ratio)
+    K = budget(w, ratio) if K is None else int(K)
     rng = _rng(w, layer, head, 1)
     protected = np.concatenate([np.arange(min(N_SINK, N)),
                                 np.arange(max(N - N_RECENT, 0), N)])
@@ -261,10 +285,20 @@ def unit_mask(w: Workload, layer: int, head: int, ratio: float) -> np.ndarray:
     raise KeyError(w.name)
 
 
-def masks(w: Workload, ratio: float, units=None) -> np.ndarray:
+def masks(w: Workload, ratio: float, units=None, schedule: str = "uniform") -> np.ndarray:
+    """Retained masks [U, N] of the given units (all by default).  schedule "uniform"
+    gives every unit the same budget; "pyramid" gives each layer its count from
+    pyramid_budgets.  The retrieval workload keeps its explicit construction."""
     if units is None:
         units = [(l, h) for l in range(w.L) for h in range(w.H)]
-    return np.stack([unit_mask(w, l, h, ratio) for (l, h) in units]).astype(np.uint8)
+    if schedule == "uniform":
+        ks = {l: None for (l, _) in units}
+    elif schedule == "pyramid":
+        pb = pyramid_budgets(w, ratio)
+        ks = {l: int(pb[l]) for (l, _) in units}
+    else:
+        raise ValueError(schedule)
+    return np.stack([unit_mask(w, l, h, ratio, ks[l]) for (l, h) in units]).astype(np.uint8)
 
 
 def random_keys(seed: int, U: int, N: int, d: int, scale: float = 1.0) -> np.ndarray:

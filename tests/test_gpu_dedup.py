@@ -100,6 +100,14 @@ def test_workload_recipes(name, over, ratio):
         assert not any(int(tw[d]) in ev for d in ev)
 
 
+def test_pyramid_budgets():
+    w = synth.get("llama", L=4, H=2, N=1500)
+    keys, _ = synth.keys(w)
+    S0 = synth.masks(w, 0.5, schedule="pyramid")
+    hl, hd, _ = run_both(keys, S0, w.L, w.H, w.tau)
+    np.testing.assert_array_equal(hd["mask"].reshape(w.units, -1).sum(1), S0.sum(1))
+
+
 @pytest.mark.parametrize("seed", range(5))
 def test_select_dedup_on_random_twin_graphs(seed):
     rng = np.random.default_rng(100 + seed)

@@ -83,6 +83,22 @@ def test_host_path_equals_device_path(chunk, pin):
     assert np.all(hn["status"] == 0)
 
 
+def test_host_path_pyramid_budgets():
+    """Per-layer budgets: every chunk carries units of different |S0|."""
+    L, H = 5, 2
+    w = synth.get("qwen", L=L, H=H, N=1024)
+    keys, _ = synth.keys(w)
+    S0 = synth.masks(w, 0.5, schedule="pyramid")
+    d = _device_run(keys, S0, L, H, w.tau, want_all=True)
+    h = _host_run(keys, S0, L, H, w.tau, True, 3, True)
+    torch.cuda.synchronize()
+    _assert_same(h, d)
+    hn = {k: v.numpy() for k, v in h.items()}
+    split_check(hn, S0, w.tau, synth.N_SINK, synth.N_RECENT)
+    np.testing.assert_array_equal(hn["mask"].reshape(L * H, -1).sum(1),
+                                  np.repeat(synth.pyramid_budgets(w, 0.5), H))
+
+
 def test_host_path_fp32_keys_and_no_scores():
     w, keys, S0 = _case("tiny", 1, 1, 512, 0.5)
     d = _device_run(keys, S0, 1, 1, w.tau, want_all=False)

@@ -180,6 +180,32 @@ def test_workload_recipes(name, over, ratio):
             assert np.all(h["mask"][u, ev] == 1)
 
 
+@pytest.mark.parametrize("name,over,ratio", [
+    ("qwen", {"L": 4, "H": 2, "N": 2048}, 0.3),     # layer 0 keeps every key
+    ("llama", {"L": 6, "H": 2, "N": 1500}, 0.5),
+    ("qwen", {"L": 3, "H": 1, "N": 2053}, 0.7),     # ragged N
+])
+def test_pyramid_budgets(name, over, ratio):
+    """Per-layer budgets in one call: every unit has its own |S0|, so the retained-first
+    column layout, the tile counts of both segments and the selection sizes differ
+    from unit to unit within the launch."""
+    w = synth.get(name, **over)
+    keys, _ = synth.keys(w)
+    S0 = synth.masks(w, ratio, schedule="pyramid")
+    k = np.repeat(synth.pyramid_budgets(w, ratio), w.H)
+    assert len(set(k.tolist())) == w.L
+    rep, h, a, r = repair_vs_oracle(keys, S0, w.L, w.H, synth.WINDOW, w.tau)
+    assert rep.n_fail == 0, rep.notes
+    assert rep.max_dev_same_twin < 1e-9
+    np.testing.assert_array_equal(h["mask"].sum(1), k)
+    full = np.flatnonzero(k == w.N)
+    for u in full:
+        # nothing evicted: b_i(S0) = b_i(all) for every row, and no swap
+        np.testing.assert_array_equal(h["score_ret"][u], h["score_all"][u])
+        np.testing.assert_array_equal(h["twin_ret"][u], h["twin_all"][u])
+        assert h["nswaps"][u] == 0
+
+
 # ---------------------------------------------------------------- selection alone
 
 @pytest.mark.parametrize("seed", range(4))
