@@ -302,8 +302,8 @@ def run_e2e(args, world, w, keys_h, mask_h, budget_h, out, stream):
     keys_p = keys_h.pin_memory()
     mask_p = mask_h.pin_memory()
     budget_p = budget_h.pin_memory()
-    chunk = args.e2e_chunk or max(1, (U + 7) // 8)
     shape = tk.shape_of(keys_p)
+    chunk = args.e2e_chunk or tk.twinkv_host_default_chunk(shape)
     arena = tk.host_arena(shape, chunk, device=stream.device)
     res = None
 
@@ -471,7 +471,8 @@ def main():
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--e2e-chunk", type=int, default=0,
-                    help="units per chunk of the host-buffer call (0: an eighth of L*H)")
+                    help="units per chunk of the host-buffer call (0: the library default, "
+                         "about an eighth of L*H aligned to whole waves of row blocks)")
     ap.add_argument("--path", choices=("repair", "dedup", "policy"), default="repair",
                     help="repair: audit + swap (the headline); dedup: the repair that "
                          "never evicts both members of a twin pair; policy: the "

@@ -218,8 +218,9 @@ twinkv_status twinkv_repair_select_noalloc(const double* score_ret, twinkv_shape
  * twinkv_repair on a cache held in host memory (for example a KV cache offloaded to the
  * host): the same audit and swap (Sec. 3.4), with every tensor argument a HOST pointer
  * of the layout above (page-locked memory lets the copies run asynchronously).  The
- * units' keys go to the device in chunks of `chunk_units` units (0: a quarter of L*H;
- * the first chunk is a quarter of that, since nothing computes while it copies in):
+ * units' keys go to the device in chunks of `chunk_units` units (0: the value
+ * twinkv_host_default_chunk returns; the first chunk is a quarter of the chunk size,
+ * since nothing computes while it copies in):
  * chunk c + 1 is copied in while the audit of chunk c runs on `stream`, and each
  * chunk's scores and twins are copied back while later chunks run.  One selection over
  * all units follows the last chunk, and S1, the swap lists, counts and statuses are
@@ -236,6 +237,12 @@ twinkv_status twinkv_repair_select_noalloc(const double* score_ret, twinkv_shape
  * ordered after each other's use of the arena.
  */
 size_t twinkv_host_arena_size(twinkv_shape s, int32_t chunk_units);
+/* The chunk size twinkv_repair_host and twinkv_host_arena_size use for chunk_units = 0
+ * on the current device: about L*H / 8 units, rounded to the nearest multiple of
+ * sms / gcd(sms, ceil(N / 128)), the number of units whose 128-row blocks fill every
+ * SM an equal number of times (so no chunk's audit ends in a partial wave), clamped
+ * to [1, L*H]; without a device, L*H / 8 unrounded.  Returns 0 for an invalid shape. */
+int32_t twinkv_host_default_chunk(twinkv_shape s);
 twinkv_status twinkv_repair_host(const void* keys, twinkv_shape s, const uint8_t* retained_mask,
                                  const int32_t* budget, float threshold,
                                  const twinkv_params* params, uint8_t* out_mask,

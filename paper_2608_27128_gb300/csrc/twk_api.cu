@@ -6,6 +6,7 @@
 #include <cstdlib>
 #include <cstring>
 #include <mutex>
+#include <numeric>
 #include <vector>
 
 #include "twinkv.h"
@@ -282,7 +283,24 @@ twinkv_status run_refine(const uint16_t* k16, const twinkv_shape& s, const float
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; }
 
 // ---- host-buffer pipeline (twinkv_repair_host) ------------------------------------
-int default_chunk_units(int U) { return U < 4 ? U : (U + 3) / 4; }
+// Units per chunk of the host path when the caller passes 0: about an eighth of the
+// units, so that later chunks' copies hide behind earlier chunks' compute, rounded to
+// the nearest multiple of the unit count whose row blocks are a whole number of waves
+// over the SMs (the persistent audit then ends no launch in a partial wave).
+int default_chunk_units(const twinkv_shape& s)
+{
+    const int U = s.L * s.H;
+    int uc = (U + 7) / 8;
+    int dev = 0, sms = 0;
+    if (cudaGetDevice(&dev) == cudaSuccess &&
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) == cudaSuccess &&
+        sms > 0) {
+        const int rb = (s.N + kBM - 1) / kBM;
+        const int step = sms / std::gcd(sms, rb);
+        if (step <= U) uc = std::max(step, (uc + step / 2) / step * step);
+    }
+    return std::max(1, std::min(uc, U));
+}
 
 struct HostArena {
     // keys: two chunk buffers; every other array covers all units
@@ -806,11 +824,16 @@ twinkv_status twinkv_repair_select_noalloc(const double* score_ret, twinkv_shape
                          out_nswaps, out_status, scratch, L, static_cast<cudaStream_t>(stream));
 }
 
+int32_t twinkv_host_default_chunk(twinkv_shape s)
+{
+    return shape_ok(s, true) ? default_chunk_units(s) : 0;
+}
+
 size_t twinkv_host_arena_size(twinkv_shape s, int32_t chunk_units)
 {
     if (!shape_ok(s, true) || chunk_units < 0) return 0;
     const int U = s.L * s.H;
-    const int uc = chunk_units == 0 ? default_chunk_units(U) : (chunk_units < U ? chunk_units : U);
+    const int uc = chunk_units == 0 ? default_chunk_units(s) : (chunk_units < U ? chunk_units : U);
     return host_arena(s, uc).total;
 }
 
@@ -830,7 +853,7 @@ twinkv_status twinkv_repair_host(const void* keys, twinkv_shape s, const uint8_t
     twinkv_status r = params_ok(p, threshold);
     if (r != TWINKV_OK) return r;
     const int U = s.L * s.H;
-    const int uc = chunk_units == 0 ? default_chunk_units(U) : (chunk_units < U ? chunk_units : U);
+    const int uc = chunk_units == 0 ? default_chunk_units(s) : (chunk_units < U ? chunk_units : U);
     const HostArena A = host_arena(s, uc);
     if (!arena || (reinterpret_cast<uintptr_t>(arena) & 255) != 0 || arena_bytes < A.total)
         return TWINKV_ERR_WORKSPACE;

@@ -32,7 +32,8 @@ EXPORTED = (
     "twinkv_workspace_size", "twinkv_redundancy", "twinkv_repair", "twinkv_repair_select",
     "twinkv_status_string", "twinkv_get_last_error", "twinkv_set_wait_timeout_ns",
     "twinkv_wait_probe", "twinkv_profile_begin", "twinkv_profile_end",
-    "twinkv_repair_select_noalloc", "twinkv_host_arena_size", "twinkv_repair_host",
+    "twinkv_repair_select_noalloc", "twinkv_host_arena_size", "twinkv_host_default_chunk",
+    "twinkv_repair_host",
     "twinkv_policy", "twinkv_repair_dedup", "twinkv_repair_select_dedup",
 )
 
@@ -94,6 +95,8 @@ def load(build_if_missing: bool = True):
                                                      _P]
         lib.twinkv_host_arena_size.argtypes = [Shape, ctypes.c_int32]
         lib.twinkv_host_arena_size.restype = ctypes.c_size_t
+        lib.twinkv_host_default_chunk.argtypes = [Shape]
+        lib.twinkv_host_default_chunk.restype = ctypes.c_int32
         lib.twinkv_repair_host.argtypes = [_P, Shape, _P, _P, ctypes.c_float,
                                            ctypes.POINTER(Params), _P, _P, _P, _P, _P, _P, _P,
                                            _P, ctypes.c_int32, _P, ctypes.c_size_t, _P]
@@ -432,6 +435,11 @@ def _out_host(t, name, dtype, shape, pin):
     if t is None:
         return torch.empty(shape, dtype=dtype, pin_memory=pin)
     return _need_host(t, name, dtype, shape)
+
+
+def twinkv_host_default_chunk(shape: Shape) -> int:
+    """Units per chunk twinkv_repair_host uses when chunk_units is 0."""
+    return int(load().twinkv_host_default_chunk(shape))
 
 
 def twinkv_host_arena_size(shape: Shape, chunk_units: int = 0) -> int:

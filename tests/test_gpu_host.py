@@ -125,6 +125,25 @@ def test_back_to_back_calls_on_a_side_stream():
     _assert_same(h2, d2)
 
 
+def test_default_chunk_fills_whole_waves():
+    """chunk_units = 0: about an eighth of the units, in whole waves of 128-row blocks
+    over the SMs, and the arena size agrees with the explicit value."""
+    import math
+    sms = torch.cuda.get_device_properties(device()).multi_processor_count
+    for L, H, N, d in [(36, 8, 16384, 128), (16, 8, 8192, 64), (1, 8, 131072, 128),
+                       (2, 3, 1500, 64), (36, 8, 32768, 128)]:
+        s = tk.Shape(L, H, N, d, tk.BF16)
+        uc = tk.twinkv_host_default_chunk(s)
+        U, rb = L * H, -(-N // 128)
+        step = sms // math.gcd(sms, rb)
+        assert 1 <= uc <= U
+        if step <= U:
+            assert uc % step == 0 and (uc * rb) % sms == 0
+            assert abs(uc - (U + 7) // 8) <= step // 2 + 1 or uc == step
+        assert tk.twinkv_host_arena_size(s, 0) == tk.twinkv_host_arena_size(s, uc)
+    assert tk.twinkv_host_default_chunk(tk.Shape(0, 8, 100, 64, tk.BF16)) == 0
+
+
 def test_arena_too_small_is_rejected():
     L, H = 1, 2
     _, keys, S0 = _case("llama", L, H, 600, 0.5)
