@@ -21,9 +21,9 @@ from paper_2608_27128_gb300 import twinkv as tk
 pytestmark = [pytest.mark.gpu, pytest.mark.slow]
 
 
-def run_full(w, ratio):
+def run_full(w, ratio, schedule="uniform"):
     keys, truths = synth.keys(w)
-    S0 = synth.masks(w, ratio)
+    S0 = synth.masks(w, ratio, schedule=schedule)
     U, N = S0.shape
     kt = keys_tensor(keys, w.L, w.H)
     mt = torch.from_numpy(S0.reshape(w.L, w.H, N)).to(device())
@@ -109,6 +109,24 @@ def test_qwen_full(ratio):
     invariants(S0, h, w.tau)
     planted(truths, h, S0)
     rep = full_units(keys, S0, h, [5], w.tau)
+    assert rep.n_fail == 0, rep.notes
+    assert rep.max_dev_same_twin < 1e-9
+
+
+def test_qwen_full_pyramid_budgets():
+    """Per-layer budgets at full size: layer 0 keeps all 16384 keys (no evicted
+    segment), the last layer keeps 6554; one launch covers them all."""
+    w = synth.get("qwen")
+    keys, truths, S0, h = run_full(w, 0.3, schedule="pyramid")
+    k = np.repeat(synth.pyramid_budgets(w, 0.3), w.H)
+    np.testing.assert_array_equal(S0.sum(1), k)
+    split_check(h, S0, w.tau, synth.N_SINK, synth.N_RECENT)
+    invariants(S0, h, w.tau)
+    planted(truths, h, S0)
+    for u in range(w.H):   # layer 0: nothing evicted
+        np.testing.assert_array_equal(h["score_ret"][u], h["score_all"][u])
+        assert h["nswaps"][u] == 0
+    rep = full_units(keys, S0, h, [1, w.units - 1], w.tau)
     assert rep.n_fail == 0, rep.notes
     assert rep.max_dev_same_twin < 1e-9
 
