@@ -218,9 +218,11 @@ twinkv_status twinkv_repair_select_noalloc(const double* score_ret, twinkv_shape
  * twinkv_repair on a cache held in host memory (for example a KV cache offloaded to the
  * host): the same audit and swap (Sec. 3.4), with every tensor argument a HOST pointer
  * of the layout above (page-locked memory lets the copies run asynchronously).  The
- * units' keys go to the device in chunks of `chunk_units` units (0: the value
- * twinkv_host_default_chunk returns; the first chunk is a quarter of the chunk size,
- * since nothing computes while it copies in):
+ * units' keys go to the device in chunks of at most `chunk_units` units (0: the value
+ * twinkv_host_default_chunk returns).  Nothing computes while the first chunk copies
+ * in and each chunk's compute has to cover the next one's copy, so the chunks grow
+ * from one unit by x2.5 (sizes of a whole wave of 128-row blocks or more rounded to
+ * the nearest multiple of such a wave) up to `chunk_units`:
  * chunk c + 1 is copied in while the audit of chunk c runs on `stream`, and each
  * chunk's scores and twins are copied back while later chunks run.  One selection over
  * all units follows the last chunk, and S1, the swap lists, counts and statuses are

@@ -287,6 +287,13 @@ bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 
 // units, so that later chunks' copies hide behind earlier chunks' compute, rounded to
 // the nearest multiple of the unit count whose row blocks are a whole number of waves
 // over the SMs (the persistent audit then ends no launch in a partial wave).
+// The number of units whose 128-row blocks fill `sms` SMs an equal number of times.
+int wave_units(const twinkv_shape& s, int sms)
+{
+    const int rb = (s.N + kBM - 1) / kBM;
+    return sms > 0 ? sms / std::gcd(sms, rb) : 0;
+}
+
 int default_chunk_units(const twinkv_shape& s)
 {
     const int U = s.L * s.H;
@@ -295,8 +302,7 @@ int default_chunk_units(const twinkv_shape& s)
     if (cudaGetDevice(&dev) == cudaSuccess &&
         cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) == cudaSuccess &&
         sms > 0) {
-        const int rb = (s.N + kBM - 1) / kBM;
-        const int step = sms / std::gcd(sms, rb);
+        const int step = wave_units(s, sms);
         if (step <= U) uc = std::max(step, (uc + step / 2) / step * step);
     }
     return std::max(1, std::min(uc, U));
@@ -880,12 +886,21 @@ twinkv_status twinkv_repair_host(const void* keys, twinkv_shape s, const uint8_t
         return TWINKV_ERR_CUDA;
     if (budget && !ck(cudaMemcpyAsync(d_budget, budget, U * 4, cudaMemcpyHostToDevice, hs->h2d)))
         return TWINKV_ERR_CUDA;
-    // The first chunk is a quarter of the others: nothing computes while it copies in.
-    const int first = uc >= 4 ? uc / 4 : uc;
+    // Nothing computes while the first chunk copies in, and each chunk's compute has to
+    // cover the next chunk's copy: the chunks grow from one unit by x2.5 (the audit of a
+    // unit takes about three times its keys' copy) up to uc, a size of uc's wave
+    // multiple or more rounded to the nearest such multiple.
+    const int step = wave_units(s, dev->sms);
+    auto next_size = [&](int prev) {
+        int n = prev <= 0 ? 1 : std::max(prev + 1, (5 * prev + 1) / 2);
+        if (n >= step && step > 0) n = std::max(step, (n + step / 2) / step * step);
+        return std::min(n, uc);
+    };
+    int want = 0;
     size_t u0 = 0;
     for (int c = 0; u0 < static_cast<size_t>(U); ++c) {
         const int b = c & 1;
-        const int want = c == 0 ? first : uc;
+        want = next_size(want);
         const int un = static_cast<int>(U - u0 < static_cast<size_t>(want) ? U - u0 : want);
         char* kbuf = base + A.keys + b * A.key_buf;
         // inputs, once the audit that last read this keys buffer is done
