@@ -201,6 +201,7 @@ __device__ __forceinline__ void scan2n(Shared& s, int co, int cd, int& po, int& 
 }
 
 constexpr int kE = 4;   // consecutive positions per thread in the streaming passes
+constexpr int kH = 4;   // items per thread per round of a digit histogram
 
 // One stable counting pass on digit (key >> shift) & 255 of n items; returns false
 // (and moves nothing) when every item has the same digit.
@@ -211,11 +212,18 @@ __device__ bool radix_pass(Shared& s, const uint64_t* kin, const int* iin, uint6
     for (int i = threadIdx.x; i < kW * 256; i += kT) (&s.warp_cnt[0][0])[i] = 0;
     if (threadIdx.x < 256) s.base[threadIdx.x] = 0;
     __syncthreads();
-    for (int c0 = 0; c0 < n; c0 += kT) {
-        const int i = c0 + threadIdx.x;
-        const int dg = i < n ? static_cast<int>((kin[i] >> shift) & 255) : 256;
-        const uint32_t peers = __match_any_sync(0xFFFFFFFFu, dg);
-        if (dg < 256 && lane == __ffs(peers) - 1) atomicAdd(&s.base[dg], __popc(peers));
+    for (int c0 = 0; c0 < n; c0 += kT * kH) {
+        int dg[kH];
+#pragma unroll
+        for (int e = 0; e < kH; ++e) {   // the loads first: kH in flight per thread
+            const int i = c0 + e * kT + threadIdx.x;
+            dg[e] = i < n ? static_cast<int>((kin[i] >> shift) & 255) : 256;
+        }
+#pragma unroll
+        for (int e = 0; e < kH; ++e) {
+            const uint32_t peers = __match_any_sync(0xFFFFFFFFu, dg[e]);
+            if (dg[e] < 256 && lane == __ffs(peers) - 1) atomicAdd(&s.base[dg[e]], __popc(peers));
+        }
     }
     __syncthreads();
     if (threadIdx.x < 32) {
@@ -287,15 +295,23 @@ __device__ void select_smallest(Shared& s, const uint64_t* kin, const int* iin, 
     for (int shift = 56; shift >= 0 && !whole; shift -= 8) {
         if (threadIdx.x < 256) s.base[threadIdx.x] = 0;
         __syncthreads();
-        for (int c0 = 0; c0 < n; c0 += kT) {
-            const int i = c0 + threadIdx.x;
-            int dg = 256;
-            if (i < n) {
-                const uint64_t key = kin[i];
-                if ((key & pmask) == prefix) dg = static_cast<int>((key >> shift) & 255);
+        for (int c0 = 0; c0 < n; c0 += kT * kH) {
+            int dg[kH];
+#pragma unroll
+            for (int e = 0; e < kH; ++e) {   // the loads first: kH in flight per thread
+                const int i = c0 + e * kT + threadIdx.x;
+                dg[e] = 256;
+                if (i < n) {
+                    const uint64_t key = kin[i];
+                    if ((key & pmask) == prefix) dg[e] = static_cast<int>((key >> shift) & 255);
+                }
             }
-            const uint32_t peers = __match_any_sync(0xFFFFFFFFu, dg);
-            if (dg < 256 && lane == __ffs(peers) - 1) atomicAdd(&s.base[dg], __popc(peers));
+#pragma unroll
+            for (int e = 0; e < kH; ++e) {
+                const uint32_t peers = __match_any_sync(0xFFFFFFFFu, dg[e]);
+                if (dg[e] < 256 && lane == __ffs(peers) - 1)
+                    atomicAdd(&s.base[dg[e]], __popc(peers));
+            }
         }
         __syncthreads();
         if (threadIdx.x < 32) digit_cut(s.base, need, s.sel_digit, s.sel_before, s.sel_count);
