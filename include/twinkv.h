@@ -222,21 +222,25 @@ twinkv_status twinkv_repair_select_noalloc(const double* score_ret, twinkv_shape
  * twinkv_host_default_chunk returns).  Nothing computes while the first chunk copies
  * in and each chunk's compute has to cover the next one's copy, so the chunks grow
  * from one unit by x2.5 (sizes of a whole wave of 128-row blocks or more rounded to
- * the nearest multiple of such a wave) up to `chunk_units`:
- * chunk c + 1 is copied in while the audit of chunk c runs on `stream`, and each
- * chunk's scores and twins are copied back while later chunks run.  One selection over
- * all units follows the last chunk, and S1, the swap lists, counts and statuses are
- * copied back after it.
+ * the nearest multiple of such a wave) up to `chunk_units`.
+ * Per chunk, ordered by events:
+ *   - its keys and mask are copied in on a copy stream the library keeps per device;
+ *   - its prefix counts, retained-first layout and audit run on `stream`;
+ *   - the exact values of its winners run on a second library stream, in blocks that
+ *     fit on the SMs beside the next chunk's audit;
+ *   - its scores and twins are copied back on a third.
+ * Three chunk buffers let chunk c + 1's copy run while chunk c - 1 is still being
+ * finished.  One selection over all units follows the last chunk, and S1,
+ * the swap lists, counts and statuses are copied back after it.
  *   arena        caller-owned DEVICE memory of twinkv_host_arena_size(s, chunk_units)
- *                bytes, 256-byte aligned: two chunk buffers of keys, the mask, b and
- *                twins of every unit, the outputs, one chunk's workspace and the
+ *                bytes, 256-byte aligned: three chunk buffers of keys and three chunk
+ *                workspaces, the mask, b and twins of every unit, the outputs and the
  *                selection's workspace.  The library allocates nothing.
  *   out_*        host outputs as in twinkv_repair (out_score_ret .. out_twin_all may be
  *                NULL); valid once `stream` has completed.  Unlike twinkv_repair, the
  *                entries of out_swaps past out_nswaps[u] are overwritten with
  *                unspecified values (the whole swap array is copied back).
- * The copies run on two streams the library keeps per device; calls on one device are
- * ordered after each other's use of the arena.
+ * Calls on one device are ordered after each other's use of the arena.
  */
 size_t twinkv_host_arena_size(twinkv_shape s, int32_t chunk_units);
 /* The chunk size twinkv_repair_host and twinkv_host_arena_size use for chunk_units = 0

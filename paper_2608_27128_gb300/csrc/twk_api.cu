@@ -274,19 +274,17 @@ twinkv_status launch_select(const twinkv_shape& s, const double* b, const uint8_
 }
 
 twinkv_status run_refine(const uint16_t* k16, const twinkv_shape& s, const float4* norm2,
-                         const int* t0, int* t1, double* b0, double* b1, cudaStream_t st)
+                         const int* t0, int* t1, double* b0, double* b1, cudaStream_t st,
+                         bool beside_audit = false)
 {
     ProfScope p(TWINKV_KERNEL_REFINE, st);
-    return cuda_status(launch_refine(k16, s.L * s.H, s.N, s.d, norm2, t0, t1, b0, b1, st));
+    return cuda_status(
+        launch_refine(k16, s.L * s.H, s.N, s.d, norm2, t0, t1, b0, b1, st, beside_audit));
 }
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; }
 
 // ---- host-buffer pipeline (twinkv_repair_host) ------------------------------------
-// Units per chunk of the host path when the caller passes 0: about an eighth of the
-// units, so that later chunks' copies hide behind earlier chunks' compute, rounded to
-// the nearest multiple of the unit count whose row blocks are a whole number of waves
-// over the SMs (the persistent audit then ends no launch in a partial wave).
 // The number of units whose 128-row blocks fill `sms` SMs an equal number of times.
 int wave_units(const twinkv_shape& s, int sms)
 {
@@ -294,6 +292,10 @@ int wave_units(const twinkv_shape& s, int sms)
     return sms > 0 ? sms / std::gcd(sms, rb) : 0;
 }
 
+// Units per chunk of the host path when the caller passes 0: about an eighth of the
+// units, so that later chunks' copies hide behind earlier chunks' compute, rounded to
+// the nearest multiple of the unit count whose row blocks are a whole number of waves
+// over the SMs (the persistent audit then ends no launch in a partial wave).
 int default_chunk_units(const twinkv_shape& s)
 {
     const int U = s.L * s.H;
@@ -308,12 +310,17 @@ int default_chunk_units(const twinkv_shape& s)
     return std::max(1, std::min(uc, U));
 }
 
+// Chunk buffers of the host path: with three, chunk c + 1's copy waits only for chunk
+// c - 2's exact values, so it runs well ahead of the audit that needs it.
+constexpr int kChunkBufs = 3;
+
 struct HostArena {
-    // keys: two chunk buffers; every other array covers all units
+    // keys and audit-stage workspaces: kChunkBufs chunk buffers each; every other array
+    // covers all units
     size_t keys = 0, mask = 0, budget = 0, bret = 0, tret = 0, sall = 0, tall = 0, omask = 0,
            oswaps = 0, onswaps = 0, ostatus = 0;
     size_t key_buf = 0;                // bytes of one keys chunk buffer
-    size_t ws = 0, ws_bytes = 0;       // audit-stage workspace of one chunk
+    size_t ws = 0, ws_bytes = 0;       // workspaces of one chunk, ws_bytes apart
     size_t sel = 0, sel_bytes = 0;     // selection workspace over all units
     size_t total = 0;
 };
@@ -330,7 +337,7 @@ HostArena host_arena(const twinkv_shape& s, int uc)
     const size_t N = static_cast<size_t>(s.N), U = static_cast<size_t>(s.L) * s.H;
     const size_t esize = s.dtype == TWINKV_F32 ? 4 : 2;
     A.key_buf = up256(static_cast<size_t>(uc) * N * s.d * esize);
-    A.keys = take(2 * A.key_buf);
+    A.keys = take(kChunkBufs * A.key_buf);
     A.mask = take(U * N);
     A.budget = take(U * 4);
     A.bret = take(U * N * 8);
@@ -344,8 +351,8 @@ HostArena host_arena(const twinkv_shape& s, int uc)
     twinkv_shape sc = s;
     sc.L = 1;
     sc.H = uc;
-    A.ws_bytes = layout(sc, TWINKV_OP_REPAIR).total;
-    A.ws = take(A.ws_bytes);
+    A.ws_bytes = up256(layout(sc, TWINKV_OP_REPAIR).total);
+    A.ws = take(kChunkBufs * A.ws_bytes);
     A.sel_bytes = layout(s, TWINKV_OP_REPAIR_SELECT).total;
     A.sel = take(A.sel_bytes);
     A.total = off;
@@ -354,8 +361,8 @@ HostArena host_arena(const twinkv_shape& s, int uc)
 
 struct HostStreams {
     bool ready = false;
-    cudaStream_t h2d = nullptr, d2h = nullptr;
-    cudaEvent_t in[2], done[2], sel, fin;
+    cudaStream_t h2d = nullptr, post = nullptr, d2h = nullptr;   // copies in; refine; copies out
+    cudaEvent_t in[kChunkBufs], aud[kChunkBufs], done[kChunkBufs], sel, fin;
 };
 HostStreams g_hs[kMaxDevices];
 
@@ -367,10 +374,12 @@ twinkv_status host_streams(HostStreams** out)
     HostStreams& h = g_hs[dev];
     if (!h.ready) {
         if (cudaStreamCreateWithFlags(&h.h2d, cudaStreamNonBlocking) != cudaSuccess ||
-            cudaStreamCreateWithFlags(&h.d2h, cudaStreamNonBlocking) != cudaSuccess)
+            cudaStreamCreateWithFlags(&h.d2h, cudaStreamNonBlocking) != cudaSuccess ||
+            cudaStreamCreateWithFlags(&h.post, cudaStreamNonBlocking) != cudaSuccess)
             return TWINKV_ERR_CUDA;
-        for (int b = 0; b < 2; ++b)
+        for (int b = 0; b < kChunkBufs; ++b)
             if (cudaEventCreateWithFlags(&h.in[b], cudaEventDisableTiming) != cudaSuccess ||
+                cudaEventCreateWithFlags(&h.aud[b], cudaEventDisableTiming) != cudaSuccess ||
                 cudaEventCreateWithFlags(&h.done[b], cudaEventDisableTiming) != cudaSuccess)
                 return TWINKV_ERR_CUDA;
         if (cudaEventCreateWithFlags(&h.sel, cudaEventDisableTiming) != cudaSuccess ||
@@ -649,14 +658,42 @@ namespace {
 // The audit stages of the repair for one set of units: bf16 keys, retained-first
 // gather, audit, exact values.  Writes b_i(S0) to bret and its twin's position to t0;
 // b_i(all) and its twin to out_score_all / out_twin_all when either is given.
-twinkv_status audit_stages(const DeviceInfo* dev, const void* keys, const twinkv_shape& s,
-                           const uint8_t* retained_mask, const twinkv_params& p, double* bret,
-                           int* t0, double* out_score_all, int32_t* out_twin_all,
-                           void* workspace, const Layout& L, cudaStream_t st)
+// The audit's inputs in `workspace`: bf16 keys (fp32 keys are rounded), the retained
+// prefix counts, and the retained-first column layout with its metadata and the norm
+// records.  *k16 receives the bf16 keys.
+twinkv_status prep_stages(const void* keys, const twinkv_shape& s, const uint8_t* retained_mask,
+                          void* workspace, const Layout& L, cudaStream_t st,
+                          const uint16_t** k16)
 {
     twinkv_status r;
-    const uint16_t* k16 = nullptr;
-    if ((r = keys_bf16(keys, s, workspace, L, st, &k16)) != TWINKV_OK) return r;
+    if ((r = keys_bf16(keys, s, workspace, L, st, k16)) != TWINKV_OK) return r;
+    const int U = s.L * s.H;
+    const int64_t NP = column_stride(s.N);
+    {
+        ProfScope pr(TWINKV_KERNEL_PREP, st);
+        if (launch_scan(retained_mask, U, s.N, at<int>(workspace, L.cnt),
+                        at<int>(workspace, L.kb), st) != cudaSuccess)
+            return TWINKV_ERR_CUDA;
+    }
+    ProfScope pr(TWINKV_KERNEL_PREP, st);
+    if (launch_gather(*k16, retained_mask, at<int>(workspace, L.cnt), at<int>(workspace, L.kb),
+                      U, s.N, s.d, NP, at<uint16_t>(workspace, L.kp),
+                      at<float>(workspace, L.colrinv), at<int>(workspace, L.colpos),
+                      at<float4>(workspace, L.norm2), st) != cudaSuccess)
+        return TWINKV_ERR_CUDA;
+    return TWINKV_OK;
+}
+
+// The audit (Eq. 4 and b_i(all)) and the exact value of each winner, on the inputs
+// prep_stages left in `workspace`.  With refine_st given, the exact values run there
+// after the audit (ordered by audit_done), in blocks that fit beside the next audit.
+twinkv_status main_stages(const DeviceInfo* dev, const uint16_t* k16, const twinkv_shape& s,
+                          const twinkv_params& p, double* bret, int* t0, double* out_score_all,
+                          int32_t* out_twin_all, void* workspace, const Layout& L,
+                          cudaStream_t st, cudaStream_t refine_st = nullptr,
+                          cudaEvent_t audit_done = nullptr)
+{
+    twinkv_status r;
     const int U = s.L * s.H;
     const int64_t NP = column_stride(s.N);
     float* colrinv = at<float>(workspace, L.colrinv);
@@ -665,16 +702,6 @@ twinkv_status audit_stages(const DeviceInfo* dev, const void* keys, const twinkv
     uint16_t* kp = at<uint16_t>(workspace, L.kp);
     int* cnt = at<int>(workspace, L.cnt);
     int* kb = at<int>(workspace, L.kb);
-    {
-        ProfScope pr(TWINKV_KERNEL_PREP, st);
-        if (launch_scan(retained_mask, U, s.N, cnt, kb, st) != cudaSuccess) return TWINKV_ERR_CUDA;
-    }
-    {
-        ProfScope pr(TWINKV_KERNEL_PREP, st);
-        if (launch_gather(k16, retained_mask, cnt, kb, U, s.N, s.d, NP, kp, colrinv, colpos,
-                          norm2, st) != cudaSuccess)
-            return TWINKV_ERR_CUDA;
-    }
     const bool need_all = out_score_all || out_twin_all;
     int* t1 = need_all ? (out_twin_all ? out_twin_all : at<int>(workspace, L.twin1)) : nullptr;
     AuditArgs a;
@@ -698,7 +725,22 @@ twinkv_status audit_stages(const DeviceInfo* dev, const void* keys, const twinkv
     a.mant_mask = 0xFFFFFFE0u;
     if ((r = run_audit(*dev, s, k16, kp, static_cast<int64_t>(U) * NP, a, st)) != TWINKV_OK)
         return r;
-    return run_refine(k16, s, norm2, t0, t1, bret, out_score_all, st);
+    if (!refine_st) return run_refine(k16, s, norm2, t0, t1, bret, out_score_all, st);
+    if (cudaEventRecord(audit_done, st) != cudaSuccess ||
+        cudaStreamWaitEvent(refine_st, audit_done, 0) != cudaSuccess)
+        return TWINKV_ERR_CUDA;
+    return run_refine(k16, s, norm2, t0, t1, bret, out_score_all, refine_st, true);
+}
+
+twinkv_status audit_stages(const DeviceInfo* dev, const void* keys, const twinkv_shape& s,
+                           const uint8_t* retained_mask, const twinkv_params& p, double* bret,
+                           int* t0, double* out_score_all, int32_t* out_twin_all,
+                           void* workspace, const Layout& L, cudaStream_t st)
+{
+    const uint16_t* k16 = nullptr;
+    const twinkv_status r = prep_stages(keys, s, retained_mask, workspace, L, st, &k16);
+    if (r != TWINKV_OK) return r;
+    return main_stages(dev, k16, s, p, bret, t0, out_score_all, out_twin_all, workspace, L, st);
 }
 
 twinkv_status repair_impl(const void* keys, twinkv_shape s, const uint8_t* retained_mask,
@@ -896,32 +938,40 @@ twinkv_status twinkv_repair_host(const void* keys, twinkv_shape s, const uint8_t
         if (n >= step && step > 0) n = std::max(step, (n + step / 2) / step * step);
         return std::min(n, uc);
     };
-    int want = 0;
+    int want = 0, last = 0;
     size_t u0 = 0;
     for (int c = 0; u0 < static_cast<size_t>(U); ++c) {
-        const int b = c & 1;
+        const int b = c % kChunkBufs;
         want = next_size(want);
         const int un = static_cast<int>(U - u0 < static_cast<size_t>(want) ? U - u0 : want);
         char* kbuf = base + A.keys + b * A.key_buf;
-        // inputs, once the audit that last read this keys buffer is done
-        if (c >= 2 && !ck(cudaStreamWaitEvent(hs->h2d, hs->done[b], 0))) return TWINKV_ERR_CUDA;
+        // inputs, once the audit and refine that last used this buffer pair are done
+        if (c >= kChunkBufs && !ck(cudaStreamWaitEvent(hs->h2d, hs->done[b], 0)))
+            return TWINKV_ERR_CUDA;
         if (!ck(cudaMemcpyAsync(kbuf, static_cast<const char*>(keys) + u0 * N * s.d * esize,
                                 un * N * s.d * esize, cudaMemcpyHostToDevice, hs->h2d)) ||
             !ck(cudaMemcpyAsync(d_mask + u0 * N, retained_mask + u0 * N, un * N,
                                 cudaMemcpyHostToDevice, hs->h2d)) ||
-            !ck(cudaEventRecord(hs->in[b], hs->h2d)))
+            !ck(cudaEventRecord(hs->in[b], hs->h2d)) ||
+            !ck(cudaStreamWaitEvent(st, hs->in[b], 0)))
             return TWINKV_ERR_CUDA;
-        // the audit stages of this chunk, into the all-unit arrays
-        if (!ck(cudaStreamWaitEvent(st, hs->in[b], 0))) return TWINKV_ERR_CUDA;
+        // Prefix counts, retained-first layout and audit of this chunk on `stream`, into
+        // this buffer's workspace and the all-unit arrays; the exact values on the
+        // refine stream, beside the next chunk's audit.
         twinkv_shape sc = s;
         sc.L = 1;
         sc.H = un;
         const Layout Lc = layout(sc, TWINKV_OP_REPAIR);
-        r = audit_stages(dev, kbuf, sc, d_mask + u0 * N, p, d_bret + u0 * N, d_tret + u0 * N,
-                         need_all ? d_sall + u0 * N : nullptr, need_all ? d_tall + u0 * N : nullptr,
-                         base + A.ws, Lc, st);
+        char* wsb = base + A.ws + b * A.ws_bytes;
+        const uint16_t* k16 = nullptr;
+        if ((r = prep_stages(kbuf, sc, d_mask + u0 * N, wsb, Lc, st, &k16)) != TWINKV_OK)
+            return r;
+        r = main_stages(dev, k16, sc, p, d_bret + u0 * N, d_tret + u0 * N,
+                        need_all ? d_sall + u0 * N : nullptr, need_all ? d_tall + u0 * N : nullptr,
+                        wsb, Lc, st, hs->post, hs->aud[b]);
         if (r != TWINKV_OK) return r;
-        if (!ck(cudaEventRecord(hs->done[b], st))) return TWINKV_ERR_CUDA;
+        if (!ck(cudaEventRecord(hs->done[b], hs->post))) return TWINKV_ERR_CUDA;
+        last = b;
         // this chunk's scores and twins go back while later chunks run
         if (!ck(cudaStreamWaitEvent(hs->d2h, hs->done[b], 0))) return TWINKV_ERR_CUDA;
         auto d2h = [&](void* dst, const void* src, size_t bytes) {
@@ -934,7 +984,9 @@ twinkv_status twinkv_repair_host(const void* keys, twinkv_shape s, const uint8_t
             return TWINKV_ERR_CUDA;
         u0 += un;
     }
-    // one selection over every unit (Sec. 3.4), then its results go back
+    // one selection over every unit (Sec. 3.4), after every chunk's exact values (the
+    // refine stream runs them in order), then its results go back
+    if (!ck(cudaStreamWaitEvent(st, hs->done[last], 0))) return TWINKV_ERR_CUDA;
     const Layout Lsel = layout(s, TWINKV_OP_REPAIR_SELECT);
     uint8_t* d_omask = reinterpret_cast<uint8_t*>(base + A.omask);
     int32_t* d_oswaps = reinterpret_cast<int32_t*>(base + A.oswaps);

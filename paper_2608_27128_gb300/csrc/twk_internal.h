@@ -85,7 +85,8 @@ cudaError_t launch_gather(const uint16_t* keys, const uint8_t* mask, const int* 
 // overwritten with the overall winner and b1 (nullable) receives its similarity.
 cudaError_t launch_refine(const uint16_t* keys, int U, int N, int d, const float4* norms,
                           const int* twin0, int* twin1, double* b0, double* b1,
-                          cudaStream_t st);
+                          cudaStream_t st,
+                          bool beside_audit = false);
 
 // audit kernel (tensor maps built by the caller)
 size_t audit_smem_bytes(int d);

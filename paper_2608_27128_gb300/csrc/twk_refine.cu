@@ -43,9 +43,11 @@ constexpr int kRowsPerBlock = kRefineThreads / kParts;
 // reach the retained best) given, the best over all columns is the larger of
 // sim(i, twin0) and sim(i, twin1), the lower position on an exact tie; twin1 is
 // overwritten with it and b1 (if given) receives its value.  Grid: (row blocks, units),
-// kParts threads per row.
-template <int D>
-__global__ void __launch_bounds__(kRefineThreads)
+// kParts threads per row.  kMinBlocks = 5 (at most 51 registers) is the standalone
+// launch; 6 caps the registers at 40 so that a block fits on an SM beside a persistent
+// audit CTA.
+template <int D, int kMinBlocks>
+__global__ void __launch_bounds__(kRefineThreads, kMinBlocks)
     refine_kernel(const uint16_t* __restrict__ keys, int N, const float4* __restrict__ norms,
                   const int* __restrict__ twin0, int* __restrict__ twin1,
                   double* __restrict__ b0, double* __restrict__ b1)
@@ -88,13 +90,17 @@ __global__ void __launch_bounds__(kRefineThreads)
 
 cudaError_t launch_refine(const uint16_t* keys, int U, int N, int d, const float4* norms,
                           const int* twin0, int* twin1, double* b0, double* b1,
-                          cudaStream_t st)
+                          cudaStream_t st, bool beside_audit)
 {
     const dim3 grid((N + kRowsPerBlock - 1) / kRowsPerBlock, U);
-    if (d == 128)
-        refine_kernel<128><<<grid, kRefineThreads, 0, st>>>(keys, N, norms, twin0, twin1, b0, b1);
+    if (d == 128 && beside_audit)
+        refine_kernel<128, 6><<<grid, kRefineThreads, 0, st>>>(keys, N, norms, twin0, twin1, b0, b1);
+    else if (d == 128)
+        refine_kernel<128, 5><<<grid, kRefineThreads, 0, st>>>(keys, N, norms, twin0, twin1, b0, b1);
+    else if (beside_audit)
+        refine_kernel<64, 6><<<grid, kRefineThreads, 0, st>>>(keys, N, norms, twin0, twin1, b0, b1);
     else
-        refine_kernel<64><<<grid, kRefineThreads, 0, st>>>(keys, N, norms, twin0, twin1, b0, b1);
+        refine_kernel<64, 5><<<grid, kRefineThreads, 0, st>>>(keys, N, norms, twin0, twin1, b0, b1);
     return cudaGetLastError();
 }
 
