@@ -349,15 +349,66 @@ __device__ void select_smallest(Shared& s, const uint64_t* kin, const int* iin, 
     __syncthreads();
 }
 
+// Lists of at most kSortMax items are sorted in shared memory (kSortMax * 12 bytes of
+// dynamic shared memory), longer ones by the radix passes over the workspace.
+constexpr int kSortMax = 4096;
+
+// Sorts the n <= kSortMax items (kin, iin) ascending by (key, position) into (kout,
+// iout), with a bitonic network in shared memory (sk, si) padded to a power of two by
+// items that sort last.  Positions are distinct, so the order equals that of a stable
+// sort by key of a list in position order.
+__device__ void smem_sort(uint64_t* sk, int* si, const uint64_t* kin, const int* iin, int n,
+                          uint64_t* kout, int* iout)
+{
+    int P = 1;
+    while (P < n) P <<= 1;
+    for (int t = threadIdx.x; t < P; t += kT) {
+        sk[t] = t < n ? kin[t] : ~0ull;
+        si[t] = t < n ? iin[t] : 0x7FFFFFFF;
+    }
+    __syncthreads();
+    for (int size = 2; size <= P; size <<= 1) {
+        for (int stride = size >> 1; stride > 0; stride >>= 1) {
+            for (int t = threadIdx.x; t < P / 2; t += kT) {
+                const int lo = 2 * t - (t & (stride - 1));
+                const int hi = lo + stride;
+                const uint64_t ka = sk[lo], kb = sk[hi];
+                const int pa = si[lo], pb = si[hi];
+                const bool gt = ka > kb || (ka == kb && pa > pb);
+                if (gt == ((lo & size) == 0)) {   // ascending blocks swap a greater first
+                    sk[lo] = kb;
+                    sk[hi] = ka;
+                    si[lo] = pb;
+                    si[hi] = pa;
+                }
+            }
+            __syncthreads();
+        }
+    }
+    for (int t = threadIdx.x; t < n; t += kT) {
+        kout[t] = sk[t];
+        iout[t] = si[t];
+    }
+    __syncthreads();
+}
+
 // The m most severe items of one list, in severity order: (key, position) pairs at
 // (k, i) with scratch (kx, ix) of the same extent; returns the position array holding
-// them.
+// them.  (sk, si): kSortMax items of shared memory.
 __device__ const int* most_severe(Shared& s, uint64_t* k, int* i, uint64_t* kx, int* ix, int n,
-                                  int m)
+                                  int m, uint64_t* sk, int* si)
 {
     if (n > m) {
         select_smallest(s, k, i, kx, ix, n, m);
+        if (m <= kSortMax) {
+            smem_sort(sk, si, kx, ix, m, k, i);
+            return i;
+        }
         return radix_sort(s, kx, ix, k, i, m) ? i : ix;
+    }
+    if (n <= kSortMax) {
+        smem_sort(sk, si, k, i, n, kx, ix);
+        return ix;
     }
     return radix_sort(s, k, i, kx, ix, n) ? ix : i;
 }
@@ -365,10 +416,22 @@ __device__ const int* most_severe(Shared& s, uint64_t* k, int* i, uint64_t* kx, 
 constexpr int kWalkChunk = 4096;   // twin ranks staged per step of the dedup walk
 
 // Dynamic shared memory of the dedup variant: 2 state bits per donor rank (n_d <= N),
-// then one chunk of staged twin ranks.
-inline size_t dedup_smem_bytes(int N)
+// then one chunk of staged twin ranks (the sort buffers follow, 16-byte aligned).
+__host__ __device__ inline size_t dedup_smem_bytes(int N)
 {
     return static_cast<size_t>((N + 15) / 16) * 4 + kWalkChunk * 4;
+}
+
+// Offset of the shared-memory sort buffers (kSortMax keys, then kSortMax positions) in
+// the dynamic shared memory, and the total dynamic bytes.
+__host__ __device__ inline size_t sort_smem_offset(bool dedup, int N)
+{
+    return dedup ? (dedup_smem_bytes(N) + 15) / 16 * 16 : 0;
+}
+
+__host__ __device__ inline size_t repair_smem_bytes(bool dedup, int N)
+{
+    return sort_smem_offset(dedup, N) + static_cast<size_t>(kSortMax) * 12;
 }
 
 template <bool kDedup>
@@ -475,19 +538,23 @@ __global__ void __launch_bounds__(kT, 2) repair_kernel(const RepairArgs a)   // 
     __syncthreads();
 
     // 4. the m most severe orphans and donors, in severity order
+    extern __shared__ __align__(16) uint32_t dyn[];
+    uint64_t* sk = reinterpret_cast<uint64_t*>(
+        reinterpret_cast<unsigned char*>(dyn) + sort_smem_offset(kDedup, N));
+    int* si = reinterpret_cast<int*>(sk + kSortMax);
     const int* orph;
     const int* don;
     int m_eff = m;
     if (!kDedup) {
-        orph = most_severe(s, k0, i0, k1, i1, n_o, m);
-        don = most_severe(s, k0 + n_o, i0 + n_o, k1 + n_o, i1 + n_o, n_d, m);
+        orph = most_severe(s, k0, i0, k1, i1, n_o, m, sk, si);
+        don = most_severe(s, k0 + n_o, i0 + n_o, k1 + n_o, i1 + n_o, n_d, m, sk, si);
     } else {
-        extern __shared__ uint32_t dyn[];
         uint32_t* state = dyn;                                   // 2 bits per rank
         int* trs = reinterpret_cast<int*>(dyn + (N + 15) / 16);  // staged twin ranks
         // every donor in severity order; the other position buffer and the key
         // buffers' donor regions are free afterwards
-        const int* spos = most_severe(s, k0 + n_o, i0 + n_o, k1 + n_o, i1 + n_o, n_d, n_d);
+        const int* spos =
+            most_severe(s, k0 + n_o, i0 + n_o, k1 + n_o, i1 + n_o, n_d, n_d, sk, si);
         int* tr = spos == i0 + n_o ? i1 + n_o : i0 + n_o;
         int* dlist = reinterpret_cast<int*>(k0 + n_o);
         int* R = a.rank_of + off;
@@ -526,7 +593,7 @@ __global__ void __launch_bounds__(kT, 2) repair_kernel(const RepairArgs a)   // 
         m_eff = acc;
         for (int j = threadIdx.x; j < m_eff; j += kT) dlist[j] = spos[dlist[j]];
         __syncthreads();
-        orph = most_severe(s, k0, i0, k1, i1, n_o, m_eff);
+        orph = most_severe(s, k0, i0, k1, i1, n_o, m_eff, sk, si);
         don = dlist;
     }
     __syncthreads();
@@ -550,11 +617,16 @@ __global__ void __launch_bounds__(kT, 2) repair_kernel(const RepairArgs a)   // 
 cudaError_t launch_repair(const RepairArgs& a, cudaStream_t st)
 {
     if (!a.twin) {
-        repair_kernel<false><<<a.U, kT, 0, st>>>(a);
+        const size_t bytes = repair_smem_bytes(false, a.N);
+        const cudaError_t e = cudaFuncSetAttribute(repair_kernel<false>,
+                                                   cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                   static_cast<int>(bytes));
+        if (e != cudaSuccess) return e;
+        repair_kernel<false><<<a.U, kT, bytes, st>>>(a);
         return cudaGetLastError();
     }
     if (a.N > kDedupMaxN) return cudaErrorInvalidValue;
-    const size_t bytes = dedup_smem_bytes(a.N);
+    const size_t bytes = repair_smem_bytes(true, a.N);
     const cudaError_t e = cudaFuncSetAttribute(
         repair_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(bytes));
     if (e != cudaSuccess) return e;
