@@ -8,13 +8,15 @@
 //      (severity key, position) pair: orphans keyed by b ascending, donors by b
 //      descending, through an order-preserving fp64 -> u64 map (-0 folded into +0);
 //   4. per list, the m most severe items: a radix select (byte histograms from the top)
-//      finds the cut, an ordered compaction keeps those items in position order, and a
-//      stable LSD radix sort (8-bit digits, warp match + per-warp digit counts; a digit
-//      position shared by every key is skipped) orders them, so equal severities keep
-//      position order (lower position first);
+//      finds the cut, an ordered compaction keeps those items in position order, and
+//      they are ordered by (key, position), so equal severities keep position order
+//      (lower position first): up to 4096 items by a bitonic network in shared memory,
+//      more by a stable LSD radix sort (8-bit digits, warp match + per-warp digit
+//      counts; a digit position shared by every key is skipped);
 //   5. m = min(|O|, |D|): S1 = S0 with the first m donors cleared and the first m
 //      orphans set; swaps[k] = (donor k, orphan k).
-// Sort buffers are caller workspace ([U][N] keys and positions, twice).
+// Sort buffers are caller workspace ([U][N] keys and positions, twice), plus 48 KB of
+// dynamic shared memory per block for the bitonic sort.
 //
 // Dedup variant (repair_kernel<true>, given the twin of every position): evicting a
 // donor keeps its twin, so a twin pair never loses both members.  All donors are
