@@ -136,6 +136,32 @@ def test_select_dedup_on_random_twin_graphs(seed):
     split_check_dedup(h, S0, 0.85, 3, 7, budget=budget)
 
 
+def test_select_dedup_with_more_than_4096_donors():
+    """All donors are sorted before the walk: more than 4096 of them takes the radix
+    passes instead of the shared-memory sort."""
+    rng = np.random.default_rng(21)
+    L, H, N = 1, 2, 20000
+    U = L * H
+    S0 = synth.random_masks(21, U, N, N // 2)
+    b = np.round(rng.uniform(0.0, 1.0, size=(U, N)), 3)
+    t = np.empty((U, N), np.int32)
+    for u in range(U):
+        ret = np.flatnonzero(S0[u])
+        t[u] = rng.choice(ret, size=N)
+        t[u][t[u] == np.arange(N)] = -1
+    out = tk.twinkv_repair_select_dedup(
+        torch.from_numpy(b.reshape(L, H, N)).to(device()),
+        torch.from_numpy(t.reshape(L, H, N)).to(device()),
+        torch.from_numpy(S0.reshape(L, H, N)).to(device()),
+        torch.from_numpy(S0.sum(1).astype(np.int32)).to(device()), threshold=0.3)
+    torch.cuda.synchronize()
+    h = {k: v.cpu().numpy() for k, v in out.items()}
+    h["score_ret"], h["twin_ret"] = b, t
+    nd = ((S0 == 1) & (b >= np.float32(0.3)))[:, 4:N - 64].sum(1)
+    assert np.all(nd > 4096), nd
+    split_check_dedup(h, S0, 0.3, synth.N_SINK, synth.N_RECENT)
+
+
 def test_size_limit_is_reported():
     N = (1 << 19) + 1
     z = torch.zeros((1, 1, N), dtype=torch.float64, device=device())

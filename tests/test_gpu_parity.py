@@ -232,6 +232,32 @@ def test_repair_select_is_bit_exact(seed):
     split_check(h, S0, tau, 4, 64, budget=budget)
 
 
+@pytest.mark.parametrize("N,frac", [(30000, 0.5), (24001, 0.35)])
+def test_repair_select_lists_on_both_sides_of_the_shared_memory_sort(N, frac):
+    """Lists of the m selected items up to 4096 are sorted in shared memory, longer ones
+    by radix passes: units with m well above and well below 4096, many equal b values
+    and ties at tau, bit-exact against the oracle's selection."""
+    rng = np.random.default_rng(N)
+    L, H = 1, 4
+    U = L * H
+    b = np.round(rng.uniform(-1.0, 1.0, size=(U, N)), 3)   # many exact ties
+    b[:, ::97] = 0.0                                          # ties at tau
+    K = np.array([N // 2, int(N * frac), N // 8, N - 64], np.int64)
+    S0 = np.zeros((U, N), np.uint8)
+    for u in range(U):
+        S0[u, rng.permutation(N)[:K[u]]] = 1
+    tau = 0.0
+    out = tk.twinkv_repair_select(
+        torch.from_numpy(b.reshape(L, H, N)).to(device()),
+        torch.from_numpy(S0.reshape(L, H, N)).to(device()),
+        torch.from_numpy(S0.sum(1).astype(np.int32)).to(device()), threshold=tau)
+    h = {k: v.cpu().numpy() for k, v in out.items()}
+    h["score_ret"] = b
+    m = h["nswaps"]
+    assert m.max() > 4096 and m.min() < 4096, m
+    split_check(h, S0, tau, 4, 64)
+
+
 def test_wait_probe_times_out_cleanly():
     assert tk.twinkv_wait_probe(2_000_000) == tk.ERR_TIMEOUT
     # the context stays usable and the sticky error word is untouched
