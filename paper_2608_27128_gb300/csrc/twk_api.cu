@@ -930,8 +930,8 @@ twinkv_status twinkv_repair_host(const void* keys, twinkv_shape s, const uint8_t
         return TWINKV_ERR_CUDA;
     // Nothing computes while the first chunk copies in, and each chunk's compute has to
     // cover the next chunk's copy: the chunks grow from one unit by x2.5 (the audit of a
-    // unit takes about three times its keys' copy) up to uc, a size of uc's wave
-    // multiple or more rounded to the nearest such multiple.
+    // unit takes about three times the copy of its keys) up to uc.  A size of one wave
+    // of units (wave_units) or more is rounded to the nearest whole number of waves.
     const int step = wave_units(s, dev->sms);
     auto next_size = [&](int prev) {
         int n = prev <= 0 ? 1 : std::max(prev + 1, (5 * prev + 1) / 2);
