@@ -1,0 +1,96 @@
+"""Register and shared-memory budgets that the launch configuration depends on, read
+from ptxas's resource report (-Xptxas -v) of an sm_103a compile of the sources.  No
+GPU is needed.
+
+- The audit kernel runs one 320-thread CTA per SM at <= 168 registers (10 warps, three
+  per scheduler) without spilling in its hot loop.
+- The refine instantiation that runs beside an audit CTA (twinkv_repair_host) must fit
+  in the registers that CTA leaves free: 168 x 320 + r x 256 <= 65536.
+- The standalone refine keeps its 48-register budget.
+- The repair kernel runs two 512-thread blocks per SM: <= 64 registers each, and its
+  static shared memory plus the 48 KB sort buffer twice within the SM's 228 KB."""
+import os
+import re
+import subprocess
+import sys
+import tempfile
+from concurrent.futures import ThreadPoolExecutor
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+sys.path.insert(0, ROOT)
+
+from paper_2608_27128_gb300 import build as B   # noqa: E402
+
+
+def _report(src):
+    """{mangled kernel name: (registers, spill store bytes, static smem bytes)}."""
+    with tempfile.TemporaryDirectory() as d:
+        p = subprocess.run([B.nvcc(), *B.ARCH, *B.FLAGS, "-Xptxas", "-v", "-c",
+                            os.path.join(B.CSRC, src), "-o", os.path.join(d, "x.o")],
+                           capture_output=True, text=True, timeout=600)
+    assert p.returncode == 0, p.stderr[-2000:]
+    out, cur = {}, None
+    for line in (p.stdout + p.stderr).splitlines():
+        m = re.search(r"Function properties for (\S+)", line)
+        if m:
+            cur = m.group(1)
+            out[cur] = [0, 0, 0]
+            continue
+        if cur is None:
+            continue
+        m = re.search(r"(\d+) bytes spill stores", line)
+        if m:
+            out[cur][1] = int(m.group(1))
+        m = re.search(r"Used (\d+) registers", line)
+        if m:
+            out[cur][0] = int(m.group(1))
+            s = re.search(r"(\d+) bytes smem", line)
+            out[cur][2] = int(s.group(1)) if s else 0
+    return out
+
+
+@pytest.fixture(scope="module")
+def reports():
+    srcs = ["twk_audit.cu", "twk_refine.cu", "twk_repair.cu"]
+    with ThreadPoolExecutor(3) as ex:
+        return dict(zip(srcs, ex.map(_report, srcs)))
+
+
+def _one(rep, pattern):
+    hits = [v for k, v in rep.items() if re.search(pattern, k)]
+    assert len(hits) == 1, (pattern, sorted(rep))
+    return hits[0]
+
+
+AUDIT_REGS = 168
+
+
+@pytest.mark.parametrize("d,count", [(128, 0), (64, 0), (128, 1), (64, 1)])
+def test_audit_kernel_budget(reports, d, count):
+    regs, spill, _ = _one(reports["twk_audit.cu"], rf"audit_kernelILi{d}ELb{count}E")
+    assert regs <= AUDIT_REGS
+    assert spill <= 8
+
+
+@pytest.mark.parametrize("d", [128, 64])
+def test_refine_beside_an_audit_cta_fits(reports, d):
+    regs, _, smem = _one(reports["twk_refine.cu"], rf"refine_kernelILi{d}ELi6E")
+    assert regs <= 40
+    assert AUDIT_REGS * 320 + regs * 256 <= 65536
+    assert smem == 0
+
+
+@pytest.mark.parametrize("d", [128, 64])
+def test_standalone_refine_budget(reports, d):
+    regs, spill, _ = _one(reports["twk_refine.cu"], rf"refine_kernelILi{d}ELi5E")
+    assert regs <= 48 and spill == 0
+
+
+@pytest.mark.parametrize("dedup", [0, 1])
+def test_repair_two_blocks_per_sm(reports, dedup):
+    regs, spill, smem = _one(reports["twk_repair.cu"], rf"repair_kernelILb{dedup}E")
+    assert regs <= 64 and spill == 0
+    # static shared memory + the 4096-item sort buffer (12 bytes per item), twice
+    assert 2 * (smem + 4096 * 12 + 1024) <= 228 * 1024
