@@ -23,7 +23,9 @@
 // a row of the warp improves its best, the chunk's column is resolved by replacing the
 // low 5 mantissa bits of each value with (31 - c) and taking one more maximum, which
 // returns the lowest column among values equal at 2^-18 relative (near-equal candidates
-// only).  Columns to ignore carry NaN (max skips
+// only; a maximum with the sign bit set takes the lowest column equal to it exactly,
+// so exact ties go to the lowest column whatever their sign).  Columns to ignore carry
+// NaN (max skips
 // NaN): padding columns have 1/||k_j|| = NaN, and window columns (|i - j| <= w) are
 // set to NaN on the few tiles that intersect the window band of the row block.
 //
@@ -162,10 +164,23 @@ __device__ __forceinline__ void fold32(const uint32_t (&x)[32], const float* rin
     const float m = tree32(v);
     const bool up = m > b.v;
     if (__any_sync(0xFFFFFFFFu, up)) {
-        float p[32];
+        // The low-bit code orders ties by lowest column only for a maximum >= +0: a
+        // negative float grows more negative as its low bits grow.  A warp where some
+        // improving row has a maximum with the sign bit set (it needs keys whose best
+        // similarity is <= 0, never the case for cache-like keys) takes the lowest
+        // column whose value equals m exactly instead.
+        const bool neg = (__float_as_uint(m) >> 31) != 0;
+        int c;
+        if (__any_sync(0xFFFFFFFFu, up && neg)) {
+            c = 31;
 #pragma unroll
-        for (int k = 0; k < 32; ++k) p[k] = pack(v[k], 31u - static_cast<uint32_t>(k), mask);
-        const int c = 31 - static_cast<int>(__float_as_uint(tree32(p)) & 31u);
+            for (int k = 30; k >= 0; --k) c = (v[k] == m) ? k : c;
+        } else {
+            float p[32];
+#pragma unroll
+            for (int k = 0; k < 32; ++k) p[k] = pack(v[k], 31u - static_cast<uint32_t>(k), mask);
+            c = 31 - static_cast<int>(__float_as_uint(tree32(p)) & 31u);
+        }
         if (up) {
             b.v = m;
             b.col = col0 + c;
@@ -279,13 +294,15 @@ __device__ __forceinline__ bool all_wait(uint64_t* bar, uint32_t parity, const W
     return __all_sync(0xFFFFFFFFu, ok);
 }
 
-// Bounded wait that ignores the abort flag (used to drain in-flight copies).
+// Bounded wait that ignores the abort flag (used to drain in-flight copies and MMAs
+// after a give-up), never shorter than kDrainFloorNs whatever the caller's limit.
 __device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity, uint64_t limit_ns)
 {
+    const uint64_t limit = limit_ns > kDrainFloorNs ? limit_ns : kDrainFloorNs;
     const uint32_t a = smem_u32(bar);
     const uint64_t t0 = globaltimer_ns();
     while (!mbar_try_wait_sleep(a, parity, 1000000u))
-        if (globaltimer_ns() - t0 > limit_ns) return;
+        if (globaltimer_ns() - t0 > limit) return;
 }
 
 // Parity of the last arming of slot s after `total` armings of a ring of `n` slots,

@@ -73,6 +73,41 @@ def test_exact_ties_go_to_lowest_position():
         assert np.all(score.cpu().numpy() == 0.0)
 
 
+def simplex(n):
+    """n keys whose pairwise similarities are all exactly -1/(n-1): the rows of a
+    Hadamard matrix of order n with the all-ones first column zeroed (each row keeps
+    n-1 entries of +-1, and two different rows have dot product 0 - 1 = -1)."""
+    h = hadamard(n)
+    h[:, 0] = 0.0
+    return h
+
+
+@pytest.mark.parametrize("n", [64, 128])
+def test_exact_negative_ties_go_to_lowest_position(n):
+    """Every candidate of every row ties at the same negative similarity: the twin is
+    the lowest position beyond the window, in both the position-order audit and the
+    retained-first audit of the repair (b_i(S0) and b_i(all)), with nothing excused."""
+    d = n
+    keys = synth.f32_to_bf16_bits(simplex(n).astype(np.float32))[None]
+    i = np.arange(n)
+    for w in (0, 5, 31):
+        score, twin = tk.twinkv_redundancy(keys_tensor(keys, 1, 1), w)
+        np.testing.assert_array_equal(twin.cpu().numpy().ravel(), np.where(i > w, 0, i + w + 1))
+        np.testing.assert_allclose(score.cpu().numpy().ravel(), -1.0 / (n - 1), rtol=0,
+                                   atol=1e-12)
+        rep, s, t = redundancy_vs_oracle(keys, 1, 1, w)
+        assert rep.n_fail == 0 and rep.n_excused == 0, rep.notes
+    S0 = synth.random_masks(n, 1, n, n // 3)
+    for w in (0, 7):
+        rep, h, a, r = repair_vs_oracle(keys, S0, 1, 1, w, 0.85, n_sink=4, n_recent=8)
+        assert rep.n_fail == 0 and rep.n_excused == 0, rep.notes
+        ret = np.flatnonzero(S0[0])
+        for row in range(n):
+            cand = ret[np.abs(ret - row) > w]
+            assert h["twin_ret"][0, row] == (cand[0] if cand.size else -1)
+            assert h["twin_all"][0, row] == (0 if row > w else row + w + 1)
+
+
 # ---------------------------------------------------------------- shape sweep
 
 REDUNDANCY_CASES = [
