@@ -66,31 +66,44 @@ def compare_best(b_gpu, t_gpu, b_orc, t_orc, b_orc2, sim, window, rows=None, S0=
     return rep
 
 
-def compare_repair(S0, S1_gpu, swaps_gpu, m_gpu, orc, b_orc, tau):
+def compare_repair(S0, S1_gpu, swaps_gpu, m_gpu, orc, b_orc, tau, n_sink=4, n_recent=64):
     """One unit's repair (S1, swap list) against the oracle run on fp64 b values.
 
     orc: oracle repair output for this unit (mask, swaps, nswaps, orphan, donor).
+    Only positions the rule can move are ever excused: evicted positions (orphan
+    candidates) and retained positions outside the protected sink and recent regions
+    (donor candidates, Sec. 3.4).  A protected retained position that changes is a
+    failure whatever its b.
     """
     rep = Report()
+    N = len(S0)
     tau_f = float(np.float32(tau))
     m_orc = int(orc["nswaps"])
-    near_tau = np.abs(b_orc - tau_f) <= BAND
+    pos = np.arange(N)
+    prot = (pos < n_sink) | (pos >= N - n_recent)
+    cand_o = S0 == 0
+    cand_d = (S0 != 0) & ~prot
+    # an orphan or donor flag that b within BAND of tau may flip
+    near_tau = (cand_o | cand_d) & (np.abs(b_orc - tau_f) <= BAND)
     excusable = near_tau.copy()
     if m_orc > 0:
         so = orc["swaps"][:m_orc, 1]
         sd = orc["swaps"][:m_orc, 0]
         cut_o, cut_d = b_orc[so[-1]], b_orc[sd[-1]]
-        cand_o = (S0 == 0)
-        cand_d = (S0 != 0)
         excusable |= cand_o & (np.abs(b_orc - cut_o) <= BAND)
         excusable |= cand_d & (np.abs(b_orc - cut_d) <= BAND)
     if m_gpu != m_orc:
-        flips = int((near_tau & ((orc["orphan"] != 0) | (orc["donor"] != 0) |
-                                 (S0 == 0) | (S0 != 0))).sum())
+        flips = int(near_tau.sum())
         if abs(m_gpu - m_orc) > flips:
             rep.fail(f"m {m_gpu} vs {m_orc}")
         else:
             rep.n_excused += 1
+            # the swaps past the shorter list follow from the flipped flags: the next
+            # donors and orphans in severity order on the side that has more
+            longer = swaps_gpu[m_orc:m_gpu] if m_gpu > m_orc else orc["swaps"][m_gpu:m_orc]
+            for d_, o_ in np.asarray(longer).reshape(-1, 2):
+                excusable[d_] |= bool(cand_d[d_])
+                excusable[o_] |= bool(cand_o[o_])
     diff = np.flatnonzero(S1_gpu != orc["mask"])
     for i in diff:
         if excusable[i]:

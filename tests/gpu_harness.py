@@ -1,4 +1,7 @@
 """Runs the CUDA path through the C ABI and scores it against the oracle."""
+import json
+import os
+
 import numpy as np
 import torch
 
@@ -67,7 +70,7 @@ def repair_vs_oracle(keys, S0, L, H, window, tau, n_sink=4, n_recent=64, want_al
     for u in range(U):
         ou = {k: r[k][u] for k in r}
         rep.add(compare_repair(S0[u], h["mask"][u], h["swaps"][u], int(h["nswaps"][u]), ou,
-                               a["b_ret"][u], tau))
+                               a["b_ret"][u], tau, n_sink, n_recent))
     split_check(h, S0, tau, n_sink, n_recent)
     assert np.all(h["status"] == 0)
     return rep, h, a, r
@@ -86,3 +89,37 @@ def split_check(h, S0, tau, n_sink, n_recent, budget=None):
         m = int(rf["nswaps"][u])
         if m > 0:
             np.testing.assert_array_equal(h["swaps"][u, :m], rf["swaps"][u, :m])
+
+
+def record(**fields):
+    """One parity record per checked configuration (failures, excused items by kind,
+    rows checked), printed and, when TWINKV_PARITY_LOG names a file, appended to it as
+    a JSON line."""
+    line = json.dumps(fields, sort_keys=True, default=float)
+    print("parity", line)
+    path = os.environ.get("TWINKV_PARITY_LOG")
+    if path:
+        with open(path, "a") as f:
+            f.write(line + "\n")
+
+
+def sampled_rows(keys, S0, h, rows_per_unit, seed, window, units=None):
+    """b_i(S0), b_i(all) and their twins of `rows_per_unit` random rows of every unit
+    (different rows in each unit) against the oracle.  Returns one Report per quantity
+    and the number of rows checked."""
+    U, N, _ = keys.shape
+    rng = np.random.default_rng(seed)
+    rep_ret, rep_all = Report(), Report()
+    n_rows = 0
+    for u in (range(U) if units is None else units):
+        rows = np.sort(rng.choice(N, size=min(rows_per_unit, N), replace=False))
+        a = oracle.audit(keys[u:u + 1], S0[u:u + 1], window=window, rows=rows)
+        sim = (lambda uu: (lambda i, j: oracle.sim(keys, uu, i, j)))(u)
+        rep_ret.add(compare_best(h["score_ret"][u, rows], h["twin_ret"][u, rows],
+                                 a["b_ret"][0], a["t_ret"][0], a["b_ret2"][0], sim, window,
+                                 rows=rows, S0=S0[u], what=f"u{u} ret"))
+        rep_all.add(compare_best(h["score_all"][u, rows], h["twin_all"][u, rows],
+                                 a["b_all"][0], a["t_all"][0], a["b_all2"][0], sim, window,
+                                 rows=rows, what=f"u{u} all"))
+        n_rows += rows.size
+    return rep_ret, rep_all, n_rows
