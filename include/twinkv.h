@@ -45,6 +45,12 @@
  * Every call only enqueues work on it and returns; outputs are valid once the stream
  * has completed.
  *
+ * Per-device state.  The first call on a device records its properties, the device
+ * addresses of the library's own device variables (its error word, the fixed scratch
+ * of twinkv_repair_select_noalloc) and, for twinkv_repair_host, three streams; they
+ * are kept until the process exits.  cudaDeviceReset on a device after the library
+ * has been called there is not supported: the recorded addresses would be stale.
+ *
  * Errors.  Argument errors that the host can see (null pointers, sizes, d, dtype,
  * window, threshold, a too-small workspace) are returned at once and nothing is
  * enqueued.  Per-unit data errors are found on the device and reported in
@@ -202,8 +208,9 @@ twinkv_status twinkv_repair_select(const double* score_ret, twinkv_shape s,
  *     same time on the GPU (for example on different streams without ordering between
  *     them) race and corrupt each other's results; order them on one stream;
  *   - the first call on each device looks up the array's device address (a host-side
- *     setup step, done once per device); make that first call before any stream
- *     capture.
+ *     setup step, done once per device and kept until the process exits, so
+ *     cudaDeviceReset after it is not supported); make that first call before any
+ *     stream capture.
  * Nothing is allocated, by this call or on its behalf.
  */
 #define TWINKV_NOALLOC_MAX_POSITIONS 262144
@@ -333,8 +340,11 @@ twinkv_status twinkv_get_last_error(void);
 
 /*
  * Upper bound, in nanoseconds, on any single device-side wait of the kernels launched
- * afterwards (default 2e9).  A wait that exceeds it makes the kernel record
- * TWINKV_ERR_TIMEOUT, release its resources and return.
+ * afterwards (default 2e9; at least 1e7, smaller values return TWINKV_ERR_INVALID_ARG
+ * and leave the limit unchanged).  A wait that exceeds it makes the kernel record
+ * TWINKV_ERR_TIMEOUT, drain the copies and tensor-core operations it already started
+ * (waiting at least 0.2 s for them, whatever this limit), release its resources and
+ * return.
  */
 twinkv_status twinkv_set_wait_timeout_ns(uint64_t ns);
 

@@ -469,7 +469,7 @@ const char* twinkv_status_string(twinkv_status st)
 
 twinkv_status twinkv_set_wait_timeout_ns(uint64_t ns)
 {
-    if (ns == 0) return TWINKV_ERR_INVALID_ARG;
+    if (ns < kMinWaitLimitNs) return TWINKV_ERR_INVALID_ARG;
     std::lock_guard<std::mutex> lk(g_mu);
     g_timeout_ns = ns;
     return TWINKV_OK;
@@ -916,6 +916,24 @@ twinkv_status twinkv_repair_host(const void* keys, twinkv_shape s, const uint8_t
     const size_t N = static_cast<size_t>(s.N);
     const size_t esize = s.dtype == TWINKV_F32 ? 4 : 2;
     auto ck = [&](cudaError_t e) { return e == cudaSuccess; };
+    // An error after work was enqueued: hs->fin is made to follow everything already
+    // queued on the three library streams and on `stream`, so that the next call, which
+    // waits on hs->fin before it reuses the arena, cannot overlap that work.  If even
+    // that fails, the streams are synchronized.
+    auto fail = [&](twinkv_status e) {
+        cudaStream_t q[3] = {hs->h2d, hs->post, st};
+        bool ok = true;
+        for (cudaStream_t x : q)
+            ok = ok && ck(cudaEventRecord(hs->sel, x)) && ck(cudaStreamWaitEvent(hs->d2h, hs->sel, 0));
+        ok = ok && ck(cudaEventRecord(hs->fin, hs->d2h));
+        if (!ok) {
+            cudaStreamSynchronize(hs->h2d);
+            cudaStreamSynchronize(hs->post);
+            cudaStreamSynchronize(hs->d2h);
+            cudaStreamSynchronize(st);
+        }
+        return e;
+    };
     uint8_t* d_mask = reinterpret_cast<uint8_t*>(base + A.mask);
     int32_t* d_budget = budget ? reinterpret_cast<int32_t*>(base + A.budget) : nullptr;
     double* d_bret = reinterpret_cast<double*>(base + A.bret);
@@ -925,9 +943,9 @@ twinkv_status twinkv_repair_host(const void* keys, twinkv_shape s, const uint8_t
     const bool need_all = out_score_all || out_twin_all;
     // A previous call's copies and selection finish before this call reuses the arena.
     if (!ck(cudaStreamWaitEvent(hs->h2d, hs->fin, 0)) || !ck(cudaStreamWaitEvent(st, hs->fin, 0)))
-        return TWINKV_ERR_CUDA;
+        return fail(TWINKV_ERR_CUDA);
     if (budget && !ck(cudaMemcpyAsync(d_budget, budget, U * 4, cudaMemcpyHostToDevice, hs->h2d)))
-        return TWINKV_ERR_CUDA;
+        return fail(TWINKV_ERR_CUDA);
     // Nothing computes while the first chunk copies in, and each chunk's compute has to
     // cover the next chunk's copy: the chunks grow from one unit by x2.5 (the audit of a
     // unit takes about three times the copy of its keys) up to uc.  A size of one wave
@@ -947,14 +965,14 @@ twinkv_status twinkv_repair_host(const void* keys, twinkv_shape s, const uint8_t
         char* kbuf = base + A.keys + b * A.key_buf;
         // inputs, once the audit and refine that last used this buffer pair are done
         if (c >= kChunkBufs && !ck(cudaStreamWaitEvent(hs->h2d, hs->done[b], 0)))
-            return TWINKV_ERR_CUDA;
+            return fail(TWINKV_ERR_CUDA);
         if (!ck(cudaMemcpyAsync(kbuf, static_cast<const char*>(keys) + u0 * N * s.d * esize,
                                 un * N * s.d * esize, cudaMemcpyHostToDevice, hs->h2d)) ||
             !ck(cudaMemcpyAsync(d_mask + u0 * N, retained_mask + u0 * N, un * N,
                                 cudaMemcpyHostToDevice, hs->h2d)) ||
             !ck(cudaEventRecord(hs->in[b], hs->h2d)) ||
             !ck(cudaStreamWaitEvent(st, hs->in[b], 0)))
-            return TWINKV_ERR_CUDA;
+            return fail(TWINKV_ERR_CUDA);
         // Prefix counts, retained-first layout and audit of this chunk on `stream`, into
         // this buffer's workspace and the all-unit arrays; the exact values on the
         // refine stream, beside the next chunk's audit.
@@ -965,15 +983,15 @@ twinkv_status twinkv_repair_host(const void* keys, twinkv_shape s, const uint8_t
         char* wsb = base + A.ws + b * A.ws_bytes;
         const uint16_t* k16 = nullptr;
         if ((r = prep_stages(kbuf, sc, d_mask + u0 * N, wsb, Lc, st, &k16)) != TWINKV_OK)
-            return r;
+            return fail(r);
         r = main_stages(dev, k16, sc, p, d_bret + u0 * N, d_tret + u0 * N,
                         need_all ? d_sall + u0 * N : nullptr, need_all ? d_tall + u0 * N : nullptr,
                         wsb, Lc, st, hs->post, hs->aud[b]);
-        if (r != TWINKV_OK) return r;
-        if (!ck(cudaEventRecord(hs->done[b], hs->post))) return TWINKV_ERR_CUDA;
+        if (r != TWINKV_OK) return fail(r);
+        if (!ck(cudaEventRecord(hs->done[b], hs->post))) return fail(TWINKV_ERR_CUDA);
         last = b;
         // this chunk's scores and twins go back while later chunks run
-        if (!ck(cudaStreamWaitEvent(hs->d2h, hs->done[b], 0))) return TWINKV_ERR_CUDA;
+        if (!ck(cudaStreamWaitEvent(hs->d2h, hs->done[b], 0))) return fail(TWINKV_ERR_CUDA);
         auto d2h = [&](void* dst, const void* src, size_t bytes) {
             return ck(cudaMemcpyAsync(dst, src, bytes, cudaMemcpyDeviceToHost, hs->d2h));
         };
@@ -981,12 +999,12 @@ twinkv_status twinkv_repair_host(const void* keys, twinkv_shape s, const uint8_t
             (out_twin_ret && !d2h(out_twin_ret + u0 * N, d_tret + u0 * N, un * N * 4)) ||
             (out_score_all && !d2h(out_score_all + u0 * N, d_sall + u0 * N, un * N * 8)) ||
             (out_twin_all && !d2h(out_twin_all + u0 * N, d_tall + u0 * N, un * N * 4)))
-            return TWINKV_ERR_CUDA;
+            return fail(TWINKV_ERR_CUDA);
         u0 += un;
     }
     // one selection over every unit (Sec. 3.4), after every chunk's exact values (the
     // refine stream runs them in order), then its results go back
-    if (!ck(cudaStreamWaitEvent(st, hs->done[last], 0))) return TWINKV_ERR_CUDA;
+    if (!ck(cudaStreamWaitEvent(st, hs->done[last], 0))) return fail(TWINKV_ERR_CUDA);
     const Layout Lsel = layout(s, TWINKV_OP_REPAIR_SELECT);
     uint8_t* d_omask = reinterpret_cast<uint8_t*>(base + A.omask);
     int32_t* d_oswaps = reinterpret_cast<int32_t*>(base + A.oswaps);
@@ -994,9 +1012,9 @@ twinkv_status twinkv_repair_host(const void* keys, twinkv_shape s, const uint8_t
     int32_t* d_ostatus = reinterpret_cast<int32_t*>(base + A.ostatus);
     if ((r = launch_select(s, d_bret, d_mask, d_budget, threshold, p, d_omask, d_oswaps,
                            d_onswaps, d_ostatus, base + A.sel, Lsel, st)) != TWINKV_OK)
-        return r;
+        return fail(r);
     if (!ck(cudaEventRecord(hs->sel, st)) || !ck(cudaStreamWaitEvent(hs->d2h, hs->sel, 0)))
-        return TWINKV_ERR_CUDA;
+        return fail(TWINKV_ERR_CUDA);
     const size_t swaps_bytes = static_cast<size_t>(U) * (N / 2) * 2 * 4;
     if (!ck(cudaMemcpyAsync(out_mask, d_omask, U * N, cudaMemcpyDeviceToHost, hs->d2h)) ||
         (out_swaps && swaps_bytes &&
@@ -1005,7 +1023,7 @@ twinkv_status twinkv_repair_host(const void* keys, twinkv_shape s, const uint8_t
         (out_status &&
          !ck(cudaMemcpyAsync(out_status, d_ostatus, U * 4, cudaMemcpyDeviceToHost, hs->d2h))) ||
         !ck(cudaEventRecord(hs->fin, hs->d2h)))
-        return TWINKV_ERR_CUDA;
+        return fail(TWINKV_ERR_CUDA);
     // The caller's stream completes only after the results reached the host.
     if (!ck(cudaStreamWaitEvent(st, hs->fin, 0))) return TWINKV_ERR_CUDA;
     return TWINKV_OK;

@@ -11,6 +11,15 @@ namespace twk {
 constexpr int kBM = 128;       // rows (keys i) per work item: the UMMA M
 constexpr int kBN = 256;       // columns (keys j) per tile: the UMMA N
 
+// Bounded waits.  A wait on work that another role of the block has to do gives up
+// after the caller's limit (twinkv_set_wait_timeout_ns, never below kMinWaitLimitNs).
+// After a give-up, the copies and MMAs a CTA already started are drained before it
+// frees its tensor memory and exits; those drain waits use at least kDrainFloorNs,
+// whatever the caller's limit, since in-flight copies and MMAs complete in
+// microseconds unless the device itself is failing.
+constexpr unsigned long long kMinWaitLimitNs = 10000000ull;    // 10 ms
+constexpr unsigned long long kDrainFloorNs = 200000000ull;     // 200 ms
+
 // Column stride of the per-unit column arrays (a multiple of kBN with room for the
 // padding of both the retained and the evicted segment).
 inline int64_t column_stride(int N) { return ((int64_t)(N + kBN - 1) / kBN) * kBN + kBN; }

@@ -105,7 +105,11 @@ def test_select_argument_errors(lib):
 
 
 def test_timeout_setting(lib):
-    assert lib.twinkv_set_wait_timeout_ns(0) == tk.ERR_INVALID_ARG
+    """Limits below 10 ms are refused on the host: with a tiny limit a CTA could give up
+    while its own copies or MMAs are still in flight."""
+    for ns in (0, 1, 1000, 9_999_999):
+        assert lib.twinkv_set_wait_timeout_ns(ns) == tk.ERR_INVALID_ARG
+    assert lib.twinkv_set_wait_timeout_ns(10_000_000) == tk.OK
     assert lib.twinkv_set_wait_timeout_ns(2_000_000_000) == tk.OK
 
 
