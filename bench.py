@@ -24,6 +24,7 @@ import os
 import statistics
 import subprocess
 import sys
+import tempfile
 import time
 
 import numpy as np
@@ -57,12 +58,19 @@ def workload_config(w, ratio, path="repair", schedule="uniform"):
             "policy": "standalone policy: counts + selection (Sec. 3.2 Eq. 2-3)"}[path]
     kbytes = w.L * w.H * w.N * w.d * 2
     per_layer = (synth.pyramid_budgets(w, ratio).tolist() if schedule == "pyramid" else None)
+    retained = synth.budget(w, ratio)
+    if w.name == "retrieval":
+        # built explicitly: 4 sinks plus the most recent positions, ceil(0.3 N) in all
+        kept = f"retains ceil(0.3 N) = {retained} keys (4 sinks + the most recent)"
+    else:
+        kept = f"ratio {ratio} (retains {retained} of {w.N} keys per head)"
     return {
         "workload": f"{WORKLOAD_NAMES[w.name]} {w.L}x{w.H}x{w.N}x{w.d} bf16 (synthetic), "
-                    f"ratio {ratio}" + (", per-layer pyramid budgets" if per_layer else "") +
+                    f"{kept}" + (", per-layer pyramid budgets" if per_layer else "") +
                     f", {what}",
         "path": path,
-        "L": w.L, "H": w.H, "N": w.N, "d": w.d, "ratio": ratio, "tau": w.tau,
+        "L": w.L, "H": w.H, "N": w.N, "d": w.d, "ratio": ratio, "retained": retained,
+        "tau": w.tau,
         "window": 32, "n_sink": 4, "n_recent": 64,
         "schedule": schedule,
         "budget_per_layer": per_layer,
@@ -81,11 +89,11 @@ class ClockSampler:
     def __init__(self, gpu_index: int):
         self.gpu = gpu_index
         self.proc = None
-        self.path = os.path.join(ROOT, "gpurun_out", f"clocks_gpu{gpu_index}.csv")
+        fd, self.path = tempfile.mkstemp(prefix=f"twinkv_clocks_gpu{gpu_index}_", suffix=".csv")
+        os.close(fd)
 
     def __enter__(self):
         try:
-            os.makedirs(os.path.dirname(self.path), exist_ok=True)
             self.f = open(self.path, "w")
             self.proc = subprocess.Popen(
                 ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}",
@@ -115,6 +123,10 @@ class ClockSampler:
                 parts = [p.strip() for p in line.split(",")]
                 if len(parts) >= 9:
                     rows.append(parts)
+        try:
+            os.remove(self.path)
+        except OSError:
+            pass
         if not rows:
             return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
         sm = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
@@ -490,10 +502,13 @@ def main():
     from paper_2608_27128_gb300 import synth
     w = synth.get(args.workload) if args.layers is None else synth.get(args.workload,
                                                                         L=args.layers)
+    # the retrieval-style cache keeps its explicit construction (4 sinks + the most
+    # recent positions, ceil(0.3 N) in all): it is labelled with that ratio
+    ratio = 0.3 if args.workload == "retrieval" else args.ratio
     if args.impl == "reference":
-        run_reference(args, w, args.ratio)
+        run_reference(args, w, ratio)
     else:
-        run_ours(args, w, args.ratio)
+        run_ours(args, w, ratio)
 
 
 if __name__ == "__main__":
