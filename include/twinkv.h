@@ -61,8 +61,10 @@
  * twinkv_get_last_error().  No call throws, traps or aborts the process.
  *
  * Precision.  The twin of each key is the argmax of fp32 tensor-core similarities
- * (bf16 products, fp32 accumulation); candidates within ~2^-16 relative of each other
- * are not told apart.  The reported b of that twin is then recomputed as
+ * (bf16 products, fp32 accumulation), the lowest position on a tie; candidates within
+ * about 8e-6 in similarity of the maximum count as tied, so such a near tie can go to
+ * a lower position than the exact argmax.  The reported b of that twin is then
+ * recomputed as
  * (k_i . k_j) / sqrt((k_i . k_i)(k_j . k_j)) with double-float dot products (relative
  * error ~1e-13) and fp64 rounding, so it is symmetric in (i, j) and exactly 1 for a
  * duplicate; orphan/donor decisions and the severity ranking use these fp64 values.

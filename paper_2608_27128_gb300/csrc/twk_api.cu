@@ -145,8 +145,9 @@ bool shape_ok(const twinkv_shape& s, bool need_d)
 size_t up256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
 
 struct Layout {
-    size_t keys16 = 0, colrinv = 0, colpos = 0, norm2 = 0, kp = 0, cnt = 0, kb = 0, twin0 = 0,
-           twin1 = 0, bret = 0, k0 = 0, i0 = 0, k1 = 0, i1 = 0, rcount = 0, rank = 0;
+    size_t keys16 = 0, colrinv = 0, colpos = 0, norm2 = 0, ukk = 0, kp = 0, cnt = 0, kb = 0,
+           twin0 = 0, twin1 = 0, bret = 0, k0 = 0, i0 = 0, k1 = 0, i1 = 0, rcount = 0,
+           rank = 0;
     size_t total = 0;
 };
 
@@ -167,6 +168,7 @@ Layout layout(const twinkv_shape& s, int op)
         L.colrinv = take(U * NP * 4);
         L.colpos = take(U * NP * 4);
         L.norm2 = take(U * N * 16);
+        if (op != TWINKV_OP_POLICY) L.ukk = take(U * 4);   // largest k.k per unit
         if (op == TWINKV_OP_REPAIR) {
             L.kp = take(U * NP * s.d * 2);
             L.cnt = take(U * N * 4);
@@ -247,7 +249,7 @@ twinkv_status launch_select(const twinkv_shape& s, const double* b, const uint8_
                             const int32_t* budget, float threshold, const twinkv_params& p,
                             uint8_t* out_mask, int32_t* out_swaps, int32_t* out_nswaps,
                             int32_t* out_status, void* ws, const Layout& L, cudaStream_t st,
-                            const int32_t* twin = nullptr)
+                            const DeviceInfo* dev, const int32_t* twin = nullptr)
 {
     RepairArgs r;
     r.U = s.L * s.H;
@@ -268,6 +270,12 @@ twinkv_status launch_select(const twinkv_shape& s, const double* b, const uint8_
     r.idx1 = at<int>(ws, L.i1);
     r.twin = twin;
     r.rank_of = twin ? at<int>(ws, L.rank) : nullptr;
+    r.cluster = select_cluster_size(r.U, r.N, dev ? dev->sms : 0);
+    if (const char* f = std::getenv("TWINKV_SELECT_CLUSTER")) {
+        // test hook: force the cluster size of the literal selection (1, 2, 4, 8, 16)
+        const int c = std::atoi(f);
+        if (c == 1 || c == 2 || c == 4 || c == 8 || c == 16) r.cluster = c;
+    }
     if (twin && s.N > kDedupMaxN) return TWINKV_ERR_UNSUPPORTED;
     ProfScope prof(TWINKV_KERNEL_REPAIR, st);
     return cuda_status(launch_repair(r, st));
@@ -571,8 +579,11 @@ twinkv_status twinkv_redundancy(const void* keys, twinkv_shape s, int32_t window
     float4* norm2 = at<float4>(workspace, L.norm2);
     {
         ProfScope p(TWINKV_KERNEL_PREP, st);
-        if (launch_norms_identity(k16, U, s.N, s.d, NP, colrinv, colpos, norm2, st) !=
-            cudaSuccess)
+        unsigned* ukk = at<unsigned>(workspace, L.ukk);
+        if (cudaMemsetAsync(ukk, 0, static_cast<size_t>(U) * 4, st) != cudaSuccess ||
+            launch_norms_identity(k16, U, s.N, s.d, NP, colrinv, colpos, norm2, st, 1.0f, ukk) !=
+                cudaSuccess ||
+            launch_scale_columns(colrinv, U, NP, ukk, st) != cudaSuccess)
             return TWINKV_ERR_CUDA;
     }
     AuditArgs a;
@@ -676,10 +687,13 @@ twinkv_status prep_stages(const void* keys, const twinkv_shape& s, const uint8_t
             return TWINKV_ERR_CUDA;
     }
     ProfScope pr(TWINKV_KERNEL_PREP, st);
-    if (launch_gather(*k16, retained_mask, at<int>(workspace, L.cnt), at<int>(workspace, L.kb),
+    unsigned* ukk = at<unsigned>(workspace, L.ukk);
+    if (cudaMemsetAsync(ukk, 0, static_cast<size_t>(U) * 4, st) != cudaSuccess ||
+        launch_gather(*k16, retained_mask, at<int>(workspace, L.cnt), at<int>(workspace, L.kb),
                       U, s.N, s.d, NP, at<uint16_t>(workspace, L.kp),
                       at<float>(workspace, L.colrinv), at<int>(workspace, L.colpos),
-                      at<float4>(workspace, L.norm2), st) != cudaSuccess)
+                      at<float4>(workspace, L.norm2), ukk, st) != cudaSuccess ||
+        launch_scale_columns(at<float>(workspace, L.colrinv), U, NP, ukk, st) != cudaSuccess)
         return TWINKV_ERR_CUDA;
     return TWINKV_OK;
 }
@@ -768,7 +782,7 @@ twinkv_status repair_impl(const void* keys, twinkv_shape s, const uint8_t* retai
                           out_twin_all, workspace, L, st)) != TWINKV_OK)
         return r;
     return launch_select(s, bret, retained_mask, budget, threshold, p, out_mask, out_swaps,
-                         out_nswaps, out_status, workspace, L, st, dedup ? t0 : nullptr);
+                         out_nswaps, out_status, workspace, L, st, dev, dedup ? t0 : nullptr);
 }
 }  // namespace
 
@@ -821,7 +835,7 @@ twinkv_status twinkv_repair_select_dedup(const double* score_ret, const int32_t*
     if ((r = device_info(&dev)) != TWINKV_OK) return r;
     return launch_select(s, score_ret, retained_mask, budget, threshold, p, out_mask, out_swaps,
                          out_nswaps, out_status, workspace, L, static_cast<cudaStream_t>(stream),
-                         twin_ret);
+                         dev, twin_ret);
 }
 
 twinkv_status twinkv_repair_select(const double* score_ret, twinkv_shape s,
@@ -843,7 +857,8 @@ twinkv_status twinkv_repair_select(const double* score_ret, twinkv_shape s,
     DeviceInfo* dev = nullptr;
     if ((r = device_info(&dev)) != TWINKV_OK) return r;
     return launch_select(s, score_ret, retained_mask, budget, threshold, p, out_mask, out_swaps,
-                         out_nswaps, out_status, workspace, L, static_cast<cudaStream_t>(stream));
+                         out_nswaps, out_status, workspace, L, static_cast<cudaStream_t>(stream),
+                         dev);
 }
 
 twinkv_status twinkv_repair_select_noalloc(const double* score_ret, twinkv_shape s,
@@ -869,7 +884,8 @@ twinkv_status twinkv_repair_select_noalloc(const double* score_ret, twinkv_shape
     if ((r = noalloc_scratch(&scratch)) != TWINKV_OK) return r;
     // The sort buffers are fully written before they are read: nothing needs clearing.
     return launch_select(s, score_ret, retained_mask, budget, threshold, p, out_mask, out_swaps,
-                         out_nswaps, out_status, scratch, L, static_cast<cudaStream_t>(stream));
+                         out_nswaps, out_status, scratch, L, static_cast<cudaStream_t>(stream),
+                         dev);
 }
 
 int32_t twinkv_host_default_chunk(twinkv_shape s)
@@ -1011,7 +1027,7 @@ twinkv_status twinkv_repair_host(const void* keys, twinkv_shape s, const uint8_t
     int32_t* d_onswaps = reinterpret_cast<int32_t*>(base + A.onswaps);
     int32_t* d_ostatus = reinterpret_cast<int32_t*>(base + A.ostatus);
     if ((r = launch_select(s, d_bret, d_mask, d_budget, threshold, p, d_omask, d_oswaps,
-                           d_onswaps, d_ostatus, base + A.sel, Lsel, st)) != TWINKV_OK)
+                           d_onswaps, d_ostatus, base + A.sel, Lsel, st, dev)) != TWINKV_OK)
         return fail(r);
     if (!ck(cudaEventRecord(hs->sel, st)) || !ck(cudaStreamWaitEvent(hs->d2h, hs->sel, 0)))
         return fail(TWINKV_ERR_CUDA);

@@ -15,17 +15,19 @@
 //   warps 2..   epilogue: four warps per column group g (kGW columns of each tile); a
 //               thread owns one row (TMEM lane) and keeps its running maximum.
 // Keys enter the tensor cores un-normalised (bf16 products are exact in fp32);
-// 1/||k_j|| is applied per element in fp32.  1/||k_i|| > 0 does not change the argmax
-// over j, so it is never applied: this kernel outputs the twin positions, and the
-// exact similarity of each chosen twin is computed afterwards (twk_refine.cu).
+// 1/||k_j|| (times a power of two per unit) is applied per element in fp32.
+// 1/||k_i|| > 0 does not change the argmax over j, so it is never applied: this kernel
+// outputs the twin positions, and the exact similarity of each chosen twin is computed
+// afterwards (twk_refine.cu).
 //
-// Max and argmax: each 32-column chunk is scaled and reduced with 3-input maxima.  When
-// a row of the warp improves its best, the chunk's column is resolved by replacing the
-// low 5 mantissa bits of each value with (31 - c) and taking one more maximum, which
-// returns the lowest column among values equal at 2^-18 relative (near-equal candidates
-// only; a maximum with the sign bit set takes the lowest column equal to it exactly,
-// so exact ties go to the lowest column whatever their sign).  Columns to ignore carry
-// NaN (max skips
+// Max and argmax: each 32-column chunk is scaled (the column scales carry a power of
+// two per unit that brings every value into [-1, 1]), offset to be positive and
+// reduced with 3-input maxima.  When a row of the warp improves its best, the chunk's
+// column is resolved by replacing the low 5 mantissa bits of each value with (31 - c)
+// and taking one more maximum, which returns the lowest column among values equal at
+// 2^-18 relative (near-equal candidates only; exact ties go to the lowest column
+// whatever their sign, as the values are never negative).  Columns to ignore carry NaN
+// (max skips
 // NaN): padding columns have 1/||k_j|| = NaN, and window columns (|i - j| <= w) are
 // set to NaN on the few tiles that intersect the window band of the row block.
 //
@@ -127,27 +129,38 @@ struct Best {
     int col;
 };
 
+// The offset added to every scaled similarity.  The column scales of a unit are
+// 2^-e_u / ||k_j||, 2^e_u above every key norm of the unit, so x_ij times the scale is
+// sim(i,j) ||k_i|| 2^-e_u, in [-1, 1]; with the offset (a little above 1, for the fp32
+// error of x_ij) every value is positive.  A compile-time constant: the fused
+// multiply-add then needs no register for it.
+constexpr float kOffset = 1.0f + 0x1p-10f;
+
 // Folds 32 columns [col0, col0 + 32) into the running best.  Each accumulator value is
-// scaled by 1/||k_j|| (NaN where the window drops the column, or where 1/||k_j|| is
-// NaN on padding) and the chunk's maximum is taken.  Only when some row of the warp
-// improves on its best (strictly, so an earlier column keeps a tie) is the column
-// resolved: each value's 5 lowest mantissa bits are replaced by (31 - column) and one
-// more maximum returns the lowest column among the values equal to the maximum at
-// 2^-18 relative.  Most chunks cost one scale and one max tree.
+// scaled and offset, v = x_ij 2^-e_u/||k_j|| + kOffset > 0, in one fused multiply-add
+// (NaN where the window drops the column, or where the column scale is NaN on
+// padding), and the chunk's maximum is taken.  Only when some row of the warp improves
+// on its best (strictly, so an earlier column keeps a tie) is the column resolved: each
+// value's 5 lowest mantissa bits are replaced by (31 - column) and one more maximum
+// returns the lowest column among the values equal to the maximum at 2^-18 relative.
+// The values are positive, where a larger low-bit code means a larger float, so ties
+// go to the lowest column whatever the sign of the similarity.  Most chunks cost one
+// fused multiply-add and one max tree.
 template <bool kMasked>
 __device__ __forceinline__ void fold32(const uint32_t (&x)[32], const float* rinv,
                                        const int* pos, int rw, uint32_t w2, uint32_t mask,
                                        int col0, Best& b)
 {
+    const float2 ofs = make_float2(kOffset, kOffset);
     float v[32];
 #pragma unroll
     for (int k = 0; k < 32; k += 4) {
         const float4 r = *reinterpret_cast<const float4*>(rinv + k);
-        const float2 p01 = __fmul2_rn(make_float2(__uint_as_float(x[k]), __uint_as_float(x[k + 1])),
-                                      make_float2(r.x, r.y));
-        const float2 p23 = __fmul2_rn(
+        const float2 p01 = __ffma2_rn(make_float2(__uint_as_float(x[k]), __uint_as_float(x[k + 1])),
+                                      make_float2(r.x, r.y), ofs);
+        const float2 p23 = __ffma2_rn(
             make_float2(__uint_as_float(x[k + 2]), __uint_as_float(x[k + 3])),
-            make_float2(r.z, r.w));
+            make_float2(r.z, r.w), ofs);
         v[k] = p01.x;
         v[k + 1] = p01.y;
         v[k + 2] = p23.x;
@@ -164,23 +177,10 @@ __device__ __forceinline__ void fold32(const uint32_t (&x)[32], const float* rin
     const float m = tree32(v);
     const bool up = m > b.v;
     if (__any_sync(0xFFFFFFFFu, up)) {
-        // The low-bit code orders ties by lowest column only for a maximum >= +0: a
-        // negative float grows more negative as its low bits grow.  A warp where some
-        // improving row has a maximum with the sign bit set (it needs keys whose best
-        // similarity is <= 0, never the case for cache-like keys) takes the lowest
-        // column whose value equals m exactly instead.
-        const bool neg = (__float_as_uint(m) >> 31) != 0;
-        int c;
-        if (__any_sync(0xFFFFFFFFu, up && neg)) {
-            c = 31;
+        float p[32];
 #pragma unroll
-            for (int k = 30; k >= 0; --k) c = (v[k] == m) ? k : c;
-        } else {
-            float p[32];
-#pragma unroll
-            for (int k = 0; k < 32; ++k) p[k] = pack(v[k], 31u - static_cast<uint32_t>(k), mask);
-            c = 31 - static_cast<int>(__float_as_uint(tree32(p)) & 31u);
-        }
+        for (int k = 0; k < 32; ++k) p[k] = pack(v[k], 31u - static_cast<uint32_t>(k), mask);
+        const int c = 31 - static_cast<int>(__float_as_uint(tree32(p)) & 31u);
         if (up) {
             b.v = m;
             b.col = col0 + c;
@@ -551,6 +551,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 
             Best b0{-INFINITY, -1}, b1{-INFINITY, -1};   // retained (or all) / evicted
             const int rw = row - w;
+
             float cnt = 0.f;                               // count mode: r_i so far
             float thr = 0.f;                               // count mode: S tau ||k_i||
             if (kCount)

@@ -66,7 +66,13 @@ struct RepairArgs {
     // dedup variant (twin != null): a donor is not evicted together with its twin
     const int* twin;            // [U][N] argmax position of b_i(S0), or null
     int* rank_of;               // [U][N] scratch: donor rank of each position
+    int cluster;                // literal variant: CTAs per unit (1, 2, 4, 8 or 16)
 };
+
+// CTAs per unit of the literal repair's selection: the largest power of two that keeps
+// all units in one wave of two CTAs per SM, slices of at least 256 positions, at most
+// 16.
+int select_cluster_size(int U, int N, int sms);
 
 // The count mode's column scales are 1/||k|| times this power of two: one saturated
 // fused multiply-add per pair then gives exactly 1 or 0 (see twk_audit.cu).
@@ -79,13 +85,20 @@ constexpr int kDedupMaxN = 1 << 19;
 cudaError_t launch_round_bf16(const float* in, uint16_t* out, int64_t n, cudaStream_t st);
 // NP must be a multiple of 64 (column_stride gives a multiple of 256).
 // rscale: a power of two that multiplies every colrinv (1 except for the count mode)
+// unit_kk (zeroed by the caller, or null): receives each unit's largest k.k.
 cudaError_t launch_norms_identity(const uint16_t* keys, int U, int N, int d, int64_t NP,
                                   float* colrinv, int* colpos, float4* norms, cudaStream_t st,
-                                  float rscale = 1.0f);
+                                  float rscale = 1.0f, unsigned* unit_kk = nullptr);
 cudaError_t launch_scan(const uint8_t* mask, int U, int N, int* cnt, int* kb, cudaStream_t st);
 cudaError_t launch_gather(const uint16_t* keys, const uint8_t* mask, const int* cnt,
                           const int* kb, int U, int N, int d, int64_t NP, uint16_t* kp,
-                          float* colrinv, int* colpos, float4* norms, cudaStream_t st);
+                          float* colrinv, int* colpos, float4* norms, unsigned* unit_kk,
+                          cudaStream_t st);
+// colrinv of every unit times 2^-e_u, 2^e_u the smallest power of two >= the unit's
+// largest ||k|| (unit_kk as written by the kernels above), so that the audit's scaled
+// similarities lie in [-1, 1] (argmax mode; not for the count mode's scales).
+cudaError_t launch_scale_columns(float* colrinv, int U, int64_t NP, const unsigned* unit_kk,
+                                 cudaStream_t st);
 
 // exact similarity of the chosen twins
 // norms[r] = {k.k hi, k.k lo, 1/||k|| hi, 1/||k|| lo} (double-float pairs) per key, as

@@ -39,15 +39,23 @@ __device__ __forceinline__ float4 key_norms(const uint16_t* key, int part, float
     return make_float4(sq.h, sq.l, rn.h, rn.l);
 }
 
+// The largest k.k of unit u so far, as float bits (k.k >= 0, so the unsigned order of
+// the bits is the float order): one atomic per warp.  Lanes pass 0 for nothing.
+__device__ __forceinline__ void unit_max_kk(unsigned* unit_kk, int64_t u, float kk)
+{
+    const unsigned m = __reduce_max_sync(0xFFFFFFFFu, __float_as_uint(kk));
+    if ((threadIdx.x & 31) == 0 && m != 0u) atomicMax(unit_kk + u, m);
+}
+
 // Mode 0 (keys as given): per column p of unit blockIdx.y, colrinv = rscale/||k_p||
 // (rscale a power of two, so the scaling is exact) and colpos = p, NaN / -1 on the
-// padding columns [N, NP); norms[u][p] = the norm record.
-// Grid (NP / kKeysPerBlock, U), kParts lanes per column.
+// padding columns [N, NP); norms[u][p] = the norm record; unit_kk[u] (if given) =
+// the unit's largest k.k.  Grid (NP / kKeysPerBlock, U), kParts lanes per column.
 template <int D>
 __global__ void __launch_bounds__(kPrepThreads)
     norms_identity_kernel(const uint16_t* __restrict__ keys, int N, int64_t NP,
                           float* __restrict__ colrinv, int* __restrict__ colpos,
-                          float4* __restrict__ norms, float rscale)
+                          float4* __restrict__ norms, float rscale, unsigned* unit_kk)
 {
     const int part = threadIdx.x % kParts;
     const int p = blockIdx.x * kKeysPerBlock + threadIdx.x / kParts;
@@ -61,6 +69,7 @@ __global__ void __launch_bounds__(kPrepThreads)
         colpos[u * NP + p] = p < N ? p : -1;
         if (p < N) norms[u * N + p] = nr;
     }
+    if (unit_kk) unit_max_kk(unit_kk, u, (part == 0 && p < N) ? nr.x : 0.f);
 }
 
 // Mode 1, step 1: cnt[u][p] = number of retained positions before p; kb[u] = |S0|.
@@ -110,13 +119,14 @@ __global__ void scan_kernel(const uint8_t* __restrict__ mask, int N, int* __rest
 // it to its column of the retained-first layout (retained keys in position order, then
 // from the next tile boundary the evicted ones), with 1/||k_p|| (fp32) and p as column
 // metadata, and writes its norm record.  Slots p >= N are the padding columns
-// [K, Kpad) and [Kpad + N - K, NP): zero keys, NaN, -1.  Grid (NP / kKeysPerBlock, U).
+// [K, Kpad) and [Kpad + N - K, NP): zero keys, NaN, -1.  unit_kk[u] = the unit's
+// largest k.k.  Grid (NP / kKeysPerBlock, U).
 template <int D>
 __global__ void __launch_bounds__(kPrepThreads)
     gather_kernel(const uint16_t* __restrict__ keys, const uint8_t* __restrict__ mask,
                   const int* __restrict__ cnt, const int* __restrict__ kb, int N, int64_t NP,
                   uint16_t* __restrict__ kp, float* __restrict__ colrinv,
-                  int* __restrict__ colpos, float4* __restrict__ norms)
+                  int* __restrict__ colpos, float4* __restrict__ norms, unsigned* unit_kk)
 {
     constexpr int Q = D / 8 / kParts;   // 16-byte chunks per lane
     const int part = threadIdx.x % kParts;
@@ -145,6 +155,25 @@ __global__ void __launch_bounds__(kPrepThreads)
         colpos[u * NP + col] = p < N ? p : -1;
         if (p < N) norms[u * N + p] = nr;
     }
+    unit_max_kk(unit_kk, u, (part == 0 && p < N) ? nr.x : 0.f);
+}
+
+// colrinv[u][c] *= 2^-e_u, the power of two with 2^e_u >= the largest ||k|| of unit u
+// (from unit_kk), so that every scaled similarity x_ij * colrinv_j = sim(i,j) ||k_i||
+// 2^-e_u lies in [-1, 1].  Exact (a power of two); NaN padding stays NaN.  A unit of
+// zero keys keeps its scale.  Grid (NP / kPrepThreads, U).
+__global__ void __launch_bounds__(kPrepThreads)
+    scale_columns_kernel(float* __restrict__ colrinv, int64_t NP,
+                         const unsigned* __restrict__ unit_kk)
+{
+    const int64_t u = blockIdx.y;
+    const int64_t c = static_cast<int64_t>(blockIdx.x) * kPrepThreads + threadIdx.x;
+    const float kk = __uint_as_float(unit_kk[u]);
+    if (c >= NP || !(kk > 0.f)) return;
+    int E;
+    (void)frexpf(kk, &E);               // kk < 2^E, so ||k|| < 2^ceil(E / 2)
+    const int e = (E + 1) >> 1;          // ceil(E / 2), also for E <= 0
+    colrinv[u * NP + c] = ldexpf(colrinv[u * NP + c], -e);
 }
 
 
@@ -161,15 +190,23 @@ cudaError_t launch_round_bf16(const float* in, uint16_t* out, int64_t n, cudaStr
 
 cudaError_t launch_norms_identity(const uint16_t* keys, int U, int N, int d, int64_t NP,
                                   float* colrinv, int* colpos, float4* norms, cudaStream_t st,
-                                  float rscale)
+                                  float rscale, unsigned* unit_kk)
 {
     const dim3 grid(static_cast<unsigned>(NP / kKeysPerBlock), U);
     if (d == 128)
         norms_identity_kernel<128><<<grid, kPrepThreads, 0, st>>>(keys, N, NP, colrinv, colpos,
-                                                                   norms, rscale);
+                                                                   norms, rscale, unit_kk);
     else
         norms_identity_kernel<64><<<grid, kPrepThreads, 0, st>>>(keys, N, NP, colrinv, colpos,
-                                                                  norms, rscale);
+                                                                  norms, rscale, unit_kk);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_scale_columns(float* colrinv, int U, int64_t NP, const unsigned* unit_kk,
+                                 cudaStream_t st)
+{
+    const dim3 grid(static_cast<unsigned>((NP + kPrepThreads - 1) / kPrepThreads), U);
+    scale_columns_kernel<<<grid, kPrepThreads, 0, st>>>(colrinv, NP, unit_kk);
     return cudaGetLastError();
 }
 
@@ -181,15 +218,16 @@ cudaError_t launch_scan(const uint8_t* mask, int U, int N, int* cnt, int* kb, cu
 
 cudaError_t launch_gather(const uint16_t* keys, const uint8_t* mask, const int* cnt,
                           const int* kb, int U, int N, int d, int64_t NP, uint16_t* kp,
-                          float* colrinv, int* colpos, float4* norms, cudaStream_t st)
+                          float* colrinv, int* colpos, float4* norms, unsigned* unit_kk,
+                          cudaStream_t st)
 {
     const dim3 grid(static_cast<unsigned>(NP / kKeysPerBlock), U);
     if (d == 128)
         gather_kernel<128><<<grid, kPrepThreads, 0, st>>>(keys, mask, cnt, kb, N, NP, kp,
-                                                           colrinv, colpos, norms);
+                                                           colrinv, colpos, norms, unit_kk);
     else
         gather_kernel<64><<<grid, kPrepThreads, 0, st>>>(keys, mask, cnt, kb, N, NP, kp,
-                                                          colrinv, colpos, norms);
+                                                          colrinv, colpos, norms, unit_kk);
     return cudaGetLastError();
 }
 

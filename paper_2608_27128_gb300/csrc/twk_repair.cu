@@ -1,32 +1,35 @@
 // twk_repair.cu -- budget-exact repair swap of TwinKV (arXiv 2608.27128, Sec. 3.4).
 //
-// One block of 512 threads per unit (layer, KV head):
-//   1. validate S0: every mask byte in {0,1}, popcount == budget (when given);
-//   2. classify  orphan = i not in S0 and b_i < tau,
-//                donor  = j in S0, outside [0, n_sink) and [N - n_recent, N), b_j >= tau;
-//   3. compact both lists in position order (warp ballots + a block scan), each entry a
-//      (severity key, position) pair: orphans keyed by b ascending, donors by b
-//      descending, through an order-preserving fp64 -> u64 map (-0 folded into +0);
-//   4. per list, the m most severe items: a radix select (byte histograms from the top)
-//      finds the cut, an ordered compaction keeps those items in position order, and
-//      they are ordered by (key, position), so equal severities keep position order
-//      (lower position first): up to 4096 items by a bitonic network in shared memory,
-//      more by a stable LSD radix sort (8-bit digits, warp match + per-warp digit
-//      counts; a digit position shared by every key is skipped);
-//   5. m = min(|O|, |D|): S1 = S0 with the first m donors cleared and the first m
-//      orphans set; swaps[k] = (donor k, orphan k).
-// Sort buffers are caller workspace ([U][N] keys and positions, twice), plus 48 KB of
-// dynamic shared memory per block for the bitonic sort.
+// Per unit (layer, KV head):
+//   classify  orphan = i not in S0 and b_i < tau,
+//             donor  = j in S0, outside [0, n_sink) and [N - n_recent, N), b_j >= tau,
+//   each entry a (severity key, position) pair: orphans keyed by b ascending, donors by
+//   b descending, through an order-preserving fp64 -> u64 map (-0 folded into +0);
+//   m = min(|O|, |D|); the m most severe orphans and donors, ordered by (key, position)
+//   so that equal severities keep position order (lower position first);
+//   S1 = S0 with the m donors cleared and the m orphans set; swaps[k] = (donor k,
+//   orphan k); a unit whose mask has a byte > 1 or whose popcount differs from its
+//   budget gets status, nswaps = -1 and S1 = S0.
 //
-// Dedup variant (repair_kernel<true>, given the twin of every position): evicting a
-// donor keeps its twin, so a twin pair never loses both members.  All donors are
-// sorted; each gets the donor rank of its twin (through a position -> rank table in
-// the workspace); one thread then walks the ranks in severity order with two bits of
-// state per rank in shared memory (evicted, pinned): a donor is skipped when it is
-// pinned (the twin of an evicted donor) or its twin is evicted, and the walk stops
-// after |O| evictions.  The ranks it needs are staged in shared memory chunk by chunk,
-// so the walk itself touches shared memory only.  m = the evictions; the m most
-// severe orphans are selected as before.
+// The literal rule (select_kernel<C>) runs each unit on a cluster of C CTAs (C = 1, 2,
+// 4, 8 or 16, chosen so that every SM has work): see "cluster selection" below.  Its
+// scratch is caller workspace ([U][N] keys and positions, twice) and 48 KB of dynamic
+// shared memory per CTA.
+//
+// Dedup variant (dedup_kernel, given the twin of every position; one 512-thread block
+// per unit): evicting a donor keeps its twin, so a twin pair never loses both members.
+// All donors are sorted; each gets the donor rank of its twin (through a position ->
+// rank table in the workspace); one thread then walks the ranks in severity order with
+// two bits of state per rank in shared memory (evicted, pinned): a donor is skipped
+// when it is pinned (the twin of an evicted donor) or its twin is evicted, and the
+// walk stops after |O| evictions.  The ranks it needs are staged in shared memory
+// chunk by chunk, so the walk itself touches shared memory only.  m = the evictions;
+// the m most severe orphans are then selected with a radix select (byte histograms
+// from the top) and sorted: up to 4096 items by a bitonic network in shared memory,
+// more by a stable LSD radix sort (8-bit digits, warp match + per-warp digit counts; a
+// digit position shared by every key is skipped).
+#include <cooperative_groups.h>
+
 #include "twk_internal.h"
 
 namespace twk {
@@ -426,18 +429,409 @@ __host__ __device__ inline size_t dedup_smem_bytes(int N)
 
 // Offset of the shared-memory sort buffers (kSortMax keys, then kSortMax positions) in
 // the dynamic shared memory, and the total dynamic bytes.
-__host__ __device__ inline size_t sort_smem_offset(bool dedup, int N)
+__host__ __device__ inline size_t sort_smem_offset(int N)
 {
-    return dedup ? (dedup_smem_bytes(N) + 15) / 16 * 16 : 0;
+    return (dedup_smem_bytes(N) + 15) / 16 * 16;
 }
 
-__host__ __device__ inline size_t repair_smem_bytes(bool dedup, int N)
+__host__ __device__ inline size_t dedup_kernel_smem_bytes(int N)
 {
-    return sort_smem_offset(dedup, N) + static_cast<size_t>(kSortMax) * 12;
+    return sort_smem_offset(N) + static_cast<size_t>(kSortMax) * 12;
 }
 
-template <bool kDedup>
-__global__ void __launch_bounds__(kT, 2) repair_kernel(const RepairArgs a)   // 2 blocks/SM
+// ---------------------------------------------------------------- cluster selection
+//
+// The literal repair (Sec. 3.4) of one unit on a cluster of C CTAs (C = 1: one CTA).
+// CTA r of the cluster owns the slice [r S, (r + 1) S) of the unit's positions.
+//   A. One pass over the slice: S1 = S0, validation counts, and the slice's orphans
+//      (forward from the slice start) and donors (backward from the slice end) as
+//      (severity key, position) pairs in keys0/idx0.  n_o + n_d never exceeds the
+//      slice length, so the two lists never meet.
+//   B. Counts through distributed shared memory: totals, this CTA's offsets, status,
+//      m = min(|O|, |D|).  The side with more than m items is cut by a radix select
+//      whose digit histograms are summed over the cluster (each CTA histograms its own
+//      items; the sums, and so every decision, are identical in every CTA); the other
+//      side is taken whole.  An ordered compaction writes the m items of each side, in
+//      position order, to keys1/idx1 (orphans at [0, m), donors at [N/2, N/2 + m)).
+//   C. Each CTA sorts its share of both lists (at most kChunk items per side) by
+//      (key, position) in shared memory; an item's place in the swap list is its rank
+//      in its own share plus, for every other share, the number of that share's items
+//      ordered before it (binary search in the other CTA's shared memory).  Larger
+//      lists are sorted by one CTA per side with the stable radix passes over the
+//      workspace.
+// Every CTA of a cluster runs the same sequence of cluster barriers: each branch and
+// loop bound that leads to one depends only on values that are identical in every CTA.
+namespace cg = cooperative_groups;
+
+constexpr int kChunk = 2048;   // items per side a CTA sorts in shared memory
+
+template <int C>
+__device__ __forceinline__ void cluster_sync()
+{
+    if constexpr (C == 1) __syncthreads();
+    else cg::this_cluster().sync();
+}
+
+// The same shared-memory object in CTA `rank` of the cluster.
+template <int C, typename T>
+__device__ __forceinline__ T* peer(T* p, int rank)
+{
+    if constexpr (C == 1) return p;
+    else return cg::this_cluster().map_shared_rank(p, rank);
+}
+
+struct ClusterShared {
+    int cnt[4];          // this CTA's orphans, donors, retained count, invalid-byte flag
+    int lcnt[2];         // compaction: this CTA's items below the cut and at it
+    int hist[2][256];    // this CTA's digit histogram, alternating between passes
+    int tot[8];          // cluster-wide values derived by thread 0
+};
+
+__device__ __forceinline__ bool before(uint64_t ka, int pa, uint64_t kb, int pb)
+{
+    return ka < kb || (ka == kb && pa < pb);
+}
+
+// Number of entries of the sorted (key, position) array of P = 2^k entries that order
+// before (k, p).
+__device__ __forceinline__ int count_before(const uint64_t* sk, const int* si, int P, uint64_t k,
+                                            int p)
+{
+    int pos = 0;
+    for (int half = P >> 1; half > 0; half >>= 1)
+        if (before(sk[pos + half - 1], si[pos + half - 1], k, p)) pos += half;
+    if (before(sk[pos], si[pos], k, p)) ++pos;
+    return pos;
+}
+
+// Slice length: ceil(N / C) rounded up to a multiple of kE.
+__host__ __device__ inline int slice_len(int N, int C)
+{
+    const int q = (N + C - 1) / C;
+    return (q + kE - 1) / kE * kE;
+}
+
+template <int C>
+__global__ void __launch_bounds__(kT, 2) select_kernel(const RepairArgs a)
+{
+    __shared__ Shared s;
+    __shared__ ClusterShared cs;
+    extern __shared__ __align__(16) uint32_t dyn[];
+    uint64_t* sk_o = reinterpret_cast<uint64_t*>(dyn);   // [kChunk] orphans' keys
+    uint64_t* sk_d = sk_o + kChunk;                      // [kChunk] donors' keys
+    int* si_o = reinterpret_cast<int*>(sk_d + kChunk);   // [kChunk] positions
+    int* si_d = si_o + kChunk;
+
+    const int tid = threadIdx.x, lane = tid & 31;
+    int r = 0;
+    if constexpr (C > 1) r = static_cast<int>(cg::this_cluster().block_rank());
+    const int u = static_cast<int>(blockIdx.x / C);
+    const int N = a.N;
+    const int64_t off = static_cast<int64_t>(u) * N;
+    const uint8_t* S0 = a.mask + off;
+    const double* b = a.b + off;
+    uint8_t* S1 = a.out_mask + off;
+    int* swaps = a.out_swaps + static_cast<int64_t>(u) * 2 * (N / 2);
+    uint64_t* K0 = a.keys0 + off;
+    int* I0 = a.idx0 + off;
+    uint64_t* K1 = a.keys1 + off;
+    int* I1 = a.idx1 + off;
+    const int S = slice_len(N, C);
+    const int lo = min(N, r * S), hi = min(N, lo + S);
+    const double tau = a.tau;
+
+    // A. S1 = S0, counts, and the slice's lists (orphans forward from lo, donors
+    // backward from hi: donor k in position order sits at hi - 1 - k)
+    int bad = 0, cnt = 0, my_o = 0, my_d = 0;
+    for (int c0 = lo; c0 < hi; c0 += kT * kE) {
+        int fo[kE], fd[kE], co = 0, cd = 0;
+        double bv[kE];
+#pragma unroll
+        for (int j = 0; j < kE; ++j) {
+            const int i = c0 + tid * kE + j;
+            fo[j] = fd[j] = 0;
+            bv[j] = 0.0;
+            if (i < hi) {
+                const uint8_t v = S0[i];
+                bv[j] = b[i];
+                S1[i] = v;
+                bad |= v > 1;
+                cnt += v != 0;
+                const bool prot = i < a.n_sink || i >= N - a.n_recent;
+                fo[j] = (v == 0 && bv[j] < tau);
+                fd[j] = (v != 0 && !prot && bv[j] >= tau);
+            }
+            co += fo[j];
+            cd += fd[j];
+        }
+        int po, pd, to, td;
+        scan2n(s, co, cd, po, pd, to, td);
+#pragma unroll
+        for (int j = 0; j < kE; ++j) {
+            const int i = c0 + tid * kE + j;
+            if (fo[j]) {
+                K0[lo + my_o + po] = ordered(bv[j]);
+                I0[lo + my_o + po] = i;
+                ++po;
+            }
+            if (fd[j]) {
+                K0[hi - 1 - (my_d + pd)] = ~ordered(bv[j]);
+                I0[hi - 1 - (my_d + pd)] = i;
+                ++pd;
+            }
+        }
+        my_o += to;
+        my_d += td;
+    }
+    if (tid < 4) s.red[tid] = 0;
+    __syncthreads();
+    bad = __reduce_or_sync(0xFFFFFFFFu, bad);
+    cnt = __reduce_add_sync(0xFFFFFFFFu, cnt);
+    if (lane == 0) {
+        atomicOr(&s.red[0], bad);
+        atomicAdd(&s.red[1], cnt);
+    }
+    __syncthreads();
+    if (tid == 0) {
+        cs.cnt[0] = my_o;
+        cs.cnt[1] = my_d;
+        cs.cnt[2] = s.red[1];
+        cs.cnt[3] = s.red[0];
+    }
+    cluster_sync<C>();
+
+    // B. totals, offsets, status and m (identical in every CTA of the cluster)
+    if (tid == 0) {
+        int n_o = 0, n_d = 0, tc = 0, tb = 0, bo = 0, bd = 0;
+        for (int q = 0; q < C; ++q) {
+            const int* rc = peer<C>(cs.cnt, q);
+            if (q == r) {
+                bo = n_o;
+                bd = n_d;
+            }
+            n_o += rc[0];
+            n_d += rc[1];
+            tc += rc[2];
+            tb |= rc[3];
+        }
+        int status = 0;
+        if (tb) status = 1;                                  // TWINKV_ERR_INVALID_ARG
+        else if (a.budget && a.budget[u] != tc) status = 3;  // TWINKV_ERR_BUDGET
+        cs.tot[0] = n_o;
+        cs.tot[1] = n_d;
+        cs.tot[2] = bo;
+        cs.tot[3] = bd;
+        cs.tot[4] = status;
+        cs.tot[5] = status ? 0 : min(n_o, n_d);
+    }
+    __syncthreads();
+    const int n_o = cs.tot[0], n_d = cs.tot[1], bo = cs.tot[2], bd = cs.tot[3];
+    const int status = cs.tot[4], m = cs.tot[5];
+    if (status != 0 || m == 0) {
+        cluster_sync<C>();   // every CTA has read the counts before any CTA exits
+        if (r == 0 && tid == 0) {
+            a.out_nswaps[u] = status ? -1 : 0;
+            if (a.out_status) a.out_status[u] = status;
+        }
+        return;
+    }
+
+    // The side with more than m items is cut (at most one: m = min(n_o, n_d)); the
+    // other is taken whole.  Item k (position order) of this CTA's list on side x:
+    auto item_key = [&](int x, int k) { return x == 0 ? K0[lo + k] : K0[hi - 1 - k]; };
+    auto item_pos = [&](int x, int k) { return x == 0 ? I0[lo + k] : I0[hi - 1 - k]; };
+    const int half = N / 2;
+    for (int x = 0; x < 2; ++x) {
+        const int mine = x == 0 ? my_o : my_d;
+        const int my_before = x == 0 ? bo : bd;
+        const int dst0 = x == 0 ? 0 : half;
+        if ((x == 0 ? n_o : n_d) == m) {
+            for (int k = tid; k < mine; k += kT) {
+                K1[dst0 + my_before + k] = item_key(x, k);
+                I1[dst0 + my_before + k] = item_pos(x, k);
+            }
+            continue;
+        }
+        // radix select of the m smallest keys over the cluster, a byte at a time from
+        // the top, stopping once the boundary bucket is taken whole
+        uint64_t prefix = 0, pmask = 0;
+        int need = m;
+        bool whole = false;
+        int pass = 0;
+        for (int shift = 56; shift >= 0 && !whole; shift -= 8, ++pass) {
+            int* h = cs.hist[pass & 1];
+            if (tid < 256) h[tid] = 0;
+            __syncthreads();
+            for (int c0 = 0; c0 < mine; c0 += kT * kH) {
+                int dg[kH];
+#pragma unroll
+                for (int e = 0; e < kH; ++e) {
+                    const int k = c0 + e * kT + tid;
+                    dg[e] = 256;
+                    if (k < mine) {
+                        const uint64_t key = item_key(x, k);
+                        if ((key & pmask) == prefix) dg[e] = static_cast<int>((key >> shift) & 255);
+                    }
+                }
+#pragma unroll
+                for (int e = 0; e < kH; ++e) {
+                    const uint32_t peers = __match_any_sync(0xFFFFFFFFu, dg[e]);
+                    if (dg[e] < 256 && lane == __ffs(peers) - 1) atomicAdd(&h[dg[e]], __popc(peers));
+                }
+            }
+            cluster_sync<C>();   // every CTA's histogram of this pass is complete
+            if (tid < 256) {
+                int t = 0;
+                for (int q = 0; q < C; ++q) t += peer<C>(h, q)[tid];
+                s.base[tid] = t;
+            }
+            __syncthreads();
+            if (tid < 32) digit_cut(s.base, need, s.sel_digit, s.sel_before, s.sel_count);
+            __syncthreads();
+            need -= s.sel_before;
+            prefix |= static_cast<uint64_t>(s.sel_digit) << shift;
+            pmask |= 255ull << shift;
+            whole = s.sel_count == need;
+            __syncthreads();
+        }
+        // ordered compaction: every item below the cut (and at it when `whole`), then
+        // the first `need` items at the cut in position order over the cluster
+        int nl = 0, ne = 0;
+        for (int k = tid; k < mine; k += kT) {
+            const uint64_t km = item_key(x, k) & pmask;
+            nl += km < prefix || (whole && km == prefix);
+            ne += !whole && km == prefix;
+        }
+        if (tid < 2) s.red[tid] = 0;
+        __syncthreads();
+        nl = __reduce_add_sync(0xFFFFFFFFu, nl);
+        ne = __reduce_add_sync(0xFFFFFFFFu, ne);
+        if (lane == 0) {
+            atomicAdd(&s.red[0], nl);
+            atomicAdd(&s.red[1], ne);
+        }
+        __syncthreads();
+        if (tid == 0) {
+            cs.lcnt[0] = s.red[0];
+            cs.lcnt[1] = s.red[1];
+        }
+        cluster_sync<C>();
+        if (tid == 0) {
+            int sel_before = 0, eq_before = 0;
+            for (int q = 0; q < r; ++q) {
+                const int* lc = peer<C>(cs.lcnt, q);
+                sel_before += lc[0] + max(0, min(lc[1], need - eq_before));
+                eq_before += lc[1];
+            }
+            cs.tot[6] = sel_before;
+            cs.tot[7] = eq_before;
+        }
+        __syncthreads();
+        int base = cs.tot[6], seen_eq = cs.tot[7];
+        for (int c0 = 0; c0 < mine; c0 += kT) {
+            const int k = c0 + tid;
+            int fl = 0, fe = 0;
+            uint64_t key = 0;
+            int pos = 0;
+            if (k < mine) {
+                key = item_key(x, k);
+                pos = item_pos(x, k);
+                const uint64_t km = key & pmask;
+                fl = km < prefix || (whole && km == prefix);
+                fe = !whole && km == prefix;
+            }
+            int pl, pe, tl, te;
+            scan2(s, fl, fe, pl, pe, tl, te);
+            const int k_eq = max(0, min(te, need - seen_eq));   // taken at the cut here
+            if (fl || (fe && pe < k_eq)) {
+                const int dst = base + pl + min(pe, k_eq);
+                K1[dst0 + dst] = key;
+                I1[dst0 + dst] = pos;
+            }
+            base += tl + k_eq;
+            seen_eq += te;
+        }
+    }
+    cluster_sync<C>();   // both lists of m items are in keys1/idx1, in position order
+
+    // C. the swap list: m items per side in severity order
+    const int q = (m + C - 1) / C;
+    if (q <= kChunk) {
+        int P = 1;
+        while (P < q) P <<= 1;
+        const int c_lo = min(m, r * q), c_n = min(m, c_lo + q) - c_lo;
+        for (int t = tid; t < P; t += kT) {
+            const bool in = t < c_n;
+            sk_o[t] = in ? K1[c_lo + t] : ~0ull;
+            si_o[t] = in ? I1[c_lo + t] : 0x7FFFFFFF;
+            sk_d[t] = in ? K1[half + c_lo + t] : ~0ull;
+            si_d[t] = in ? I1[half + c_lo + t] : 0x7FFFFFFF;
+        }
+        __syncthreads();
+        for (int size = 2; size <= P; size <<= 1) {
+            for (int stride = size >> 1; stride > 0; stride >>= 1) {
+                for (int t = tid; t < P; t += kT) {   // t < P/2: orphans, else donors
+                    const int side = t >= P / 2;
+                    const int tt = side ? t - P / 2 : t;
+                    uint64_t* sk = side ? sk_d : sk_o;
+                    int* si = side ? si_d : si_o;
+                    const int lo2 = 2 * tt - (tt & (stride - 1));
+                    const int hi2 = lo2 + stride;
+                    const uint64_t ka = sk[lo2], kb = sk[hi2];
+                    const int pa = si[lo2], pb = si[hi2];
+                    const bool gt = ka > kb || (ka == kb && pa > pb);
+                    if (gt == ((lo2 & size) == 0)) {
+                        sk[lo2] = kb;
+                        sk[hi2] = ka;
+                        si[lo2] = pb;
+                        si[hi2] = pa;
+                    }
+                }
+                __syncthreads();
+            }
+        }
+        cluster_sync<C>();   // every share is sorted
+        for (int t = tid; t < 2 * c_n; t += kT) {
+            const int side = t >= c_n;
+            const int tt = side ? t - c_n : t;
+            const uint64_t* sk = side ? sk_d : sk_o;
+            const int* si = side ? si_d : si_o;
+            const uint64_t key = sk[tt];
+            const int pos = si[tt];
+            // its rank: its place in its own share plus, in every other share, the
+            // number of items ordered before it
+            int rank = tt;
+            for (int qq = 0; qq < C; ++qq)
+                if (qq != r)
+                    rank += count_before(peer<C>(const_cast<uint64_t*>(sk), qq),
+                                         peer<C>(const_cast<int*>(si), qq), P, key, pos);
+            swaps[2 * rank + (side ? 0 : 1)] = pos;
+            S1[pos] = side ? 0 : 1;
+        }
+        cluster_sync<C>();   // every lookup into this CTA's shares is done
+    } else {
+        // long lists: one CTA per side sorts its m items with the stable radix passes
+        // (keys0/idx0, free by now, as the second buffer)
+        for (int x = 0; x < 2; ++x) {
+            if (r != (C > 1 ? x : 0)) continue;
+            const int o = x == 0 ? 0 : half;
+            const int cur = radix_sort(s, K1 + o, I1 + o, K0 + o, I0 + o, m);
+            const int* ip = (cur == 0 ? I1 : I0) + o;
+            for (int k = tid; k < m; k += kT) {
+                const int pos = ip[k];
+                swaps[2 * k + (x == 0 ? 1 : 0)] = pos;
+                S1[pos] = x == 0 ? 1 : 0;
+            }
+            __syncthreads();
+        }
+    }
+    if (r == 0 && tid == 0) {
+        a.out_nswaps[u] = m;
+        if (a.out_status) a.out_status[u] = 0;
+    }
+}
+
+__global__ void __launch_bounds__(kT, 2) dedup_kernel(const RepairArgs a)   // 2 blocks/SM
 {
     __shared__ Shared s;
     const int u = blockIdx.x;
@@ -542,15 +936,12 @@ __global__ void __launch_bounds__(kT, 2) repair_kernel(const RepairArgs a)   // 
     // 4. the m most severe orphans and donors, in severity order
     extern __shared__ __align__(16) uint32_t dyn[];
     uint64_t* sk = reinterpret_cast<uint64_t*>(
-        reinterpret_cast<unsigned char*>(dyn) + sort_smem_offset(kDedup, N));
+        reinterpret_cast<unsigned char*>(dyn) + sort_smem_offset(N));
     int* si = reinterpret_cast<int*>(sk + kSortMax);
     const int* orph;
     const int* don;
     int m_eff = m;
-    if (!kDedup) {
-        orph = most_severe(s, k0, i0, k1, i1, n_o, m, sk, si);
-        don = most_severe(s, k0 + n_o, i0 + n_o, k1 + n_o, i1 + n_o, n_d, m, sk, si);
-    } else {
+    {
         uint32_t* state = dyn;                                   // 2 bits per rank
         int* trs = reinterpret_cast<int*>(dyn + (N + 15) / 16);  // staged twin ranks
         // every donor in severity order; the other position buffer and the key
@@ -616,23 +1007,97 @@ __global__ void __launch_bounds__(kT, 2) repair_kernel(const RepairArgs a)   // 
 
 }  // namespace
 
+namespace {
+
+template <int C>
+cudaError_t config_select(const RepairArgs& a, cudaStream_t st, cudaLaunchConfig_t& cfg,
+                          cudaLaunchAttribute* at)
+{
+    const size_t bytes = 2 * static_cast<size_t>(kChunk) * 12;
+    cudaError_t e = cudaFuncSetAttribute(select_kernel<C>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         static_cast<int>(bytes));
+    if (e != cudaSuccess) return e;
+    if (C > 8) {
+        e = cudaFuncSetAttribute(select_kernel<C>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+        if (e != cudaSuccess) return e;
+    }
+    cfg = cudaLaunchConfig_t{};
+    cfg.gridDim = dim3(static_cast<unsigned>(a.U) * C);
+    cfg.blockDim = dim3(kT);
+    cfg.dynamicSmemBytes = bytes;
+    cfg.stream = st;
+    at[0].id = cudaLaunchAttributeClusterDimension;
+    at[0].val.clusterDim.x = C;
+    at[0].val.clusterDim.y = 1;
+    at[0].val.clusterDim.z = 1;
+    cfg.attrs = at;
+    cfg.numAttrs = C > 1 ? 1 : 0;   // one CTA per unit: a plain launch
+    return cudaSuccess;
+}
+
+// Launches select_kernel<C> if a cluster of C CTAs can be resident; *launched says
+// whether it was.
+template <int C>
+cudaError_t try_select(const RepairArgs& a, cudaStream_t st, bool* launched)
+{
+    *launched = false;
+    cudaLaunchConfig_t cfg;
+    cudaLaunchAttribute at[1];
+    cudaError_t e = config_select<C>(a, st, cfg, at);
+    if (e != cudaSuccess) return e;
+    if (C > 1) {
+        int clusters = 0;
+        e = cudaOccupancyMaxActiveClusters(&clusters, select_kernel<C>, &cfg);
+        if (e != cudaSuccess || clusters < 1) {
+            cudaGetLastError();   // not resident: the caller tries a smaller cluster
+            return cudaSuccess;
+        }
+    }
+    e = cudaLaunchKernelEx(&cfg, select_kernel<C>, a);
+    *launched = e == cudaSuccess;
+    return e;
+}
+
+}  // namespace
+
+int select_cluster_size(int U, int N, int sms)
+{
+    // the largest cluster that keeps every unit in one wave of two CTAs per SM (more
+    // CTAs than that queue behind each other), slices of at least 256 positions, at
+    // most 16 CTAs
+    int C = 1;
+    while (C < 16 && static_cast<int64_t>(U) * (2 * C) <= 2LL * sms && N / (2 * C) >= 256)
+        C <<= 1;
+    return C;
+}
+
 cudaError_t launch_repair(const RepairArgs& a, cudaStream_t st)
 {
     if (!a.twin) {
-        const size_t bytes = repair_smem_bytes(false, a.N);
-        const cudaError_t e = cudaFuncSetAttribute(repair_kernel<false>,
-                                                   cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                   static_cast<int>(bytes));
-        if (e != cudaSuccess) return e;
-        repair_kernel<false><<<a.U, kT, bytes, st>>>(a);
-        return cudaGetLastError();
+        int C = a.cluster;
+        cudaError_t e = cudaSuccess;
+        bool done = false;
+        while (!done) {
+            switch (C) {
+            case 16: e = try_select<16>(a, st, &done); break;
+            case 8: e = try_select<8>(a, st, &done); break;
+            case 4: e = try_select<4>(a, st, &done); break;
+            case 2: e = try_select<2>(a, st, &done); break;
+            default: e = try_select<1>(a, st, &done); C = 1; break;
+            }
+            if (e != cudaSuccess) return e;
+            if (!done && C == 1) return cudaErrorLaunchFailure;
+            C >>= 1;
+        }
+        return cudaSuccess;
     }
     if (a.N > kDedupMaxN) return cudaErrorInvalidValue;
-    const size_t bytes = repair_smem_bytes(true, a.N);
+    const size_t bytes = dedup_kernel_smem_bytes(a.N);
     const cudaError_t e = cudaFuncSetAttribute(
-        repair_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(bytes));
+        dedup_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(bytes));
     if (e != cudaSuccess) return e;
-    repair_kernel<true><<<a.U, kT, bytes, st>>>(a);
+    dedup_kernel<<<a.U, kT, bytes, st>>>(a);
     return cudaGetLastError();
 }
 

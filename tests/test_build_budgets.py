@@ -7,8 +7,9 @@ GPU is needed.
 - The refine instantiation that runs beside an audit CTA (twinkv_repair_host) must fit
   in the registers that CTA leaves free: 168 x 320 + r x 256 <= 65536.
 - The standalone refine keeps its 48-register budget.
-- The repair kernel runs two 512-thread blocks per SM: <= 64 registers each, and its
-  static shared memory plus the 48 KB sort buffer twice within the SM's 228 KB."""
+- The repair kernels (the dedup variant and every cluster size of the literal
+  selection) run two 512-thread blocks per SM: <= 64 registers each, and their static
+  shared memory plus the 48 KB of sort buffers twice within the SM's 228 KB."""
 import os
 import re
 import subprocess
@@ -88,9 +89,16 @@ def test_standalone_refine_budget(reports, d):
     assert regs <= 48 and spill == 0
 
 
-@pytest.mark.parametrize("dedup", [0, 1])
-def test_repair_two_blocks_per_sm(reports, dedup):
-    regs, spill, smem = _one(reports["twk_repair.cu"], rf"repair_kernelILb{dedup}E")
+def test_dedup_repair_two_blocks_per_sm(reports):
+    regs, spill, smem = _one(reports["twk_repair.cu"], r"dedup_kernel")
     assert regs <= 64 and spill == 0
     # static shared memory + the 4096-item sort buffer (12 bytes per item), twice
     assert 2 * (smem + 4096 * 12 + 1024) <= 228 * 1024
+
+
+@pytest.mark.parametrize("cluster", [1, 2, 4, 8, 16])
+def test_selection_two_blocks_per_sm(reports, cluster):
+    regs, spill, smem = _one(reports["twk_repair.cu"], rf"select_kernelILi{cluster}EE")
+    assert regs <= 64 and spill == 0
+    # static shared memory + two 2048-item sort shares (12 bytes per item), twice
+    assert 2 * (smem + 2 * 2048 * 12 + 1024) <= 228 * 1024

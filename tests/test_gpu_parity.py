@@ -293,6 +293,34 @@ def test_repair_select_lists_on_both_sides_of_the_shared_memory_sort(N, frac):
     split_check(h, S0, tau, 4, 64)
 
 
+@pytest.mark.parametrize("cluster", [1, 2, 4, 8, 16])
+@pytest.mark.parametrize("N,K,tau", [(30000, 15000, 0.0), (24001, 8400, 0.25), (611, 300, 0.0),
+                                     (50, 25, 0.0)])
+def test_repair_select_every_cluster_size(cluster, N, K, tau, monkeypatch):
+    """The literal selection on clusters of 1 to 16 CTAs per unit (forced; the library
+    picks the size from the unit count): lists cut on either side, shares of the swap
+    list above and below the per-CTA shared-memory sort (2048 items), slices that are
+    empty, many equal b values and ties at tau, bit-exact against the oracle."""
+    monkeypatch.setenv("TWINKV_SELECT_CLUSTER", str(cluster))
+    rng = np.random.default_rng([N, K, cluster])
+    L, H = 1, 3
+    U = L * H
+    b = np.round(rng.uniform(-1.0, 1.0, size=(U, N)), 3)   # many exact ties
+    b[:, ::89] = tau                                          # ties at tau
+    S0 = np.zeros((U, N), np.uint8)
+    for u, k in enumerate((K, N - K, N // 7)):
+        S0[u, rng.permutation(N)[:k]] = 1
+    budget = S0.sum(1).astype(np.int32)
+    out = tk.twinkv_repair_select(
+        torch.from_numpy(b.reshape(L, H, N)).to(device()),
+        torch.from_numpy(S0.reshape(L, H, N)).to(device()),
+        torch.from_numpy(budget).to(device()), threshold=tau)
+    h = {k: v.cpu().numpy() for k, v in out.items()}
+    h["score_ret"] = b
+    assert np.all(h["status"] == 0)
+    split_check(h, S0, tau, 4, 64)
+
+
 def test_wait_probe_times_out_cleanly():
     assert tk.twinkv_wait_probe(2_000_000) == tk.ERR_TIMEOUT
     # the context stays usable and the sticky error word is untouched
