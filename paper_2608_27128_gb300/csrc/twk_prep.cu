@@ -40,11 +40,21 @@ __device__ __forceinline__ float4 key_norms(const uint16_t* key, int part, float
 }
 
 // The largest k.k of unit u so far, as float bits (k.k >= 0, so the unsigned order of
-// the bits is the float order): one atomic per warp.  Lanes pass 0 for nothing.
+// the bits is the float order): one atomic per block (hundreds of blocks share a unit's
+// word, so per-warp atomics queue up).  Every thread of the block calls it; lanes pass
+// 0 for nothing.
 __device__ __forceinline__ void unit_max_kk(unsigned* unit_kk, int64_t u, float kk)
 {
+    __shared__ unsigned wmax[kPrepThreads / 32];
     const unsigned m = __reduce_max_sync(0xFFFFFFFFu, __float_as_uint(kk));
-    if ((threadIdx.x & 31) == 0 && m != 0u) atomicMax(unit_kk + u, m);
+    if ((threadIdx.x & 31) == 0) wmax[threadIdx.x >> 5] = m;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        unsigned t = 0u;
+#pragma unroll
+        for (int w = 0; w < kPrepThreads / 32; ++w) t = max(t, wmax[w]);
+        if (t != 0u) atomicMax(unit_kk + u, t);
+    }
 }
 
 // Mode 0 (keys as given): per column p of unit blockIdx.y, colrinv = rscale/||k_p||

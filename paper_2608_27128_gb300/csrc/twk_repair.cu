@@ -454,11 +454,11 @@ __host__ __device__ inline size_t dedup_kernel_smem_bytes(int N)
 //      side is taken whole.  An ordered compaction writes the m items of each side, in
 //      position order, to keys1/idx1 (orphans at [0, m), donors at [N/2, N/2 + m)).
 //   C. Each CTA sorts its share of both lists (at most kChunk items per side) by
-//      (key, position) in shared memory; an item's place in the swap list is its rank
-//      in its own share plus, for every other share, the number of that share's items
-//      ordered before it (binary search in the other CTA's shared memory).  Larger
-//      lists are sorted by one CTA per side with the stable radix passes over the
-//      workspace.
+//      (key, position) with a bitonic network in shared memory; an item's place in the
+//      swap list is its rank in its own share plus, for every other share, the number
+//      of that share's items ordered before it (binary search in the other CTA's
+//      shared memory).  Larger lists are sorted by one CTA per side with the stable
+//      radix passes over the workspace.
 // Every CTA of a cluster runs the same sequence of cluster barriers: each branch and
 // loop bound that leads to one depends only on values that are identical in every CTA.
 namespace cg = cooperative_groups;
@@ -504,11 +504,13 @@ __device__ __forceinline__ int count_before(const uint64_t* sk, const int* si, i
     return pos;
 }
 
-// Slice length: ceil(N / C) rounded up to a multiple of kE.
+constexpr int kEA = 8;   // consecutive positions per thread in the classification pass
+
+// Slice length: ceil(N / C) rounded up to a multiple of kEA.
 __host__ __device__ inline int slice_len(int N, int C)
 {
     const int q = (N + C - 1) / C;
-    return (q + kE - 1) / kE * kE;
+    return (q + kEA - 1) / kEA * kEA;
 }
 
 template <int C>
@@ -541,34 +543,64 @@ __global__ void __launch_bounds__(kT, 2) select_kernel(const RepairArgs a)
     const double tau = a.tau;
 
     // A. S1 = S0, counts, and the slice's lists (orphans forward from lo, donors
-    // backward from hi: donor k in position order sits at hi - 1 - k)
+    // backward from hi: donor k in position order sits at hi - 1 - k).  A thread takes
+    // kEA consecutive positions: one 8-byte mask load and four 16-byte b loads when
+    // every unit's rows are aligned for them (N a multiple of 8, aligned base
+    // pointers), else one at a time.
     int bad = 0, cnt = 0, my_o = 0, my_d = 0;
-    for (int c0 = lo; c0 < hi; c0 += kT * kE) {
-        int fo[kE], fd[kE], co = 0, cd = 0;
-        double bv[kE];
+    const bool vec = (N % kEA) == 0 && (reinterpret_cast<uintptr_t>(a.mask) & 7) == 0 &&
+                     (reinterpret_cast<uintptr_t>(a.out_mask) & 7) == 0 &&
+                     (reinterpret_cast<uintptr_t>(a.b) & 15) == 0;
+    for (int c0 = lo; c0 < hi; c0 += kT * kEA) {
+        const int i0 = c0 + tid * kEA;
+        uint32_t mv[kEA];
+        double bv[kEA];
+        if (vec && i0 + kEA <= hi) {
+            const uint2 m8 = *reinterpret_cast<const uint2*>(S0 + i0);
+            *reinterpret_cast<uint2*>(S1 + i0) = m8;
 #pragma unroll
-        for (int j = 0; j < kE; ++j) {
-            const int i = c0 + tid * kE + j;
-            fo[j] = fd[j] = 0;
-            bv[j] = 0.0;
-            if (i < hi) {
-                const uint8_t v = S0[i];
-                bv[j] = b[i];
-                S1[i] = v;
-                bad |= v > 1;
-                cnt += v != 0;
-                const bool prot = i < a.n_sink || i >= N - a.n_recent;
-                fo[j] = (v == 0 && bv[j] < tau);
-                fd[j] = (v != 0 && !prot && bv[j] >= tau);
+            for (int j = 0; j < 4; ++j) {
+                mv[j] = (m8.x >> (8 * j)) & 255u;
+                mv[4 + j] = (m8.y >> (8 * j)) & 255u;
             }
+            const double2* b2 = reinterpret_cast<const double2*>(b + i0);
+#pragma unroll
+            for (int j = 0; j < kEA / 2; ++j) {
+                const double2 t = b2[j];
+                bv[2 * j] = t.x;
+                bv[2 * j + 1] = t.y;
+            }
+        } else {
+#pragma unroll
+            for (int j = 0; j < kEA; ++j) {
+                const int i = i0 + j;
+                mv[j] = 0u;
+                bv[j] = 0.0;
+                if (i < hi) {
+                    mv[j] = S0[i];
+                    bv[j] = b[i];
+                    S1[i] = static_cast<uint8_t>(mv[j]);
+                }
+            }
+        }
+        int fo[kEA], fd[kEA], co = 0, cd = 0;
+#pragma unroll
+        for (int j = 0; j < kEA; ++j) {
+            const int i = i0 + j;
+            const bool in = i < hi;
+            bad |= mv[j] > 1u;
+            cnt += mv[j] != 0u;
+            const bool prot = i < a.n_sink || i >= N - a.n_recent;
+            fo[j] = in && mv[j] == 0u && bv[j] < tau;
+            fd[j] = in && mv[j] != 0u && !prot && bv[j] >= tau;
             co += fo[j];
             cd += fd[j];
         }
         int po, pd, to, td;
         scan2n(s, co, cd, po, pd, to, td);
 #pragma unroll
-        for (int j = 0; j < kE; ++j) {
-            const int i = c0 + tid * kE + j;
+        for (int j = 0; j < kEA; ++j) {
+            const int i = i0 + j;
             if (fo[j]) {
                 K0[lo + my_o + po] = ordered(bv[j]);
                 I0[lo + my_o + po] = i;
@@ -1013,7 +1045,7 @@ template <int C>
 cudaError_t config_select(const RepairArgs& a, cudaStream_t st, cudaLaunchConfig_t& cfg,
                           cudaLaunchAttribute* at)
 {
-    const size_t bytes = 2 * static_cast<size_t>(kChunk) * 12;
+    const size_t bytes = 2 * static_cast<size_t>(kChunk) * 12;   // the two shares
     cudaError_t e = cudaFuncSetAttribute(select_kernel<C>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(bytes));
