@@ -360,7 +360,8 @@ def kernel_bytes(path, U, N, d, m_total):
     if path == "policy":
         return {"prep": U * (N * d * 2 + 8 * NP + 16 * N),          # norms, identity layout
                 "repair": U * (4 * N + N)}                             # counts in, mask out
-    return {"prep": U * (5 * N + N + N * d * 2 + NP * d * 2 + 8 * NP + 16 * N),   # scan + gather
+    return {"prep": U * (5 * N + N + N * d * 2 + NP * d * 2 + 16 * NP + 16 * N),  # scan, gather,
+                                                                                   # column scaling
             "repair": U * (8 * N + N + N) + 8 * m_total,               # b, S0 in; S1 out; swaps
             "refine": U * N * (2 * d + 40)}                            # k_i, norms, twins, scores
 
