@@ -55,7 +55,10 @@ def workload_config(w, ratio, path="repair", schedule="uniform"):
     from paper_2608_27128_gb300 import synth
     what = {"repair": "audit + repair (Sec. 3.4)",
             "dedup": "audit + repair that keeps one member of each twin pair (Sec. 3.4)",
-            "policy": "standalone policy: counts + selection (Sec. 3.2 Eq. 2-3)"}[path]
+            "policy": "standalone policy: counts + selection (Sec. 3.2 Eq. 2-3)",
+            "redundancy": "b_i(all) and twins alone (Sec. 3.2), every tile",
+            "symmetric": "b_i(all) and twins alone (Sec. 3.2) from the upper-triangle "
+                         "tiles"}[path]
     kbytes = w.L * w.H * w.N * w.d * 2
     per_layer = (synth.pyramid_budgets(w, ratio).tolist() if schedule == "pyramid" else None)
     retained = synth.budget(w, ratio)
@@ -251,6 +254,10 @@ def run_ours(args, w, ratio):
     ws = tk.workspace(shape, tk.OP_REPAIR, dev)
     out = None
 
+    if args.path == "redundancy":
+        ws = tk.workspace(shape, tk.OP_REDUNDANCY, dev)
+    elif args.path == "symmetric":
+        ws = tk.workspace(shape, tk.OP_REDUNDANCY_SYMMETRIC, dev)
     if args.path == "policy":
         ws = tk.workspace(shape, tk.OP_POLICY, dev)
         if args.schedule == "pyramid":
@@ -260,7 +267,11 @@ def run_ours(args, w, ratio):
 
     def step(k=keys, m=mask, b=budget):
         nonlocal out
-        if args.path == "policy":
+        if args.path == "redundancy":
+            out = tk.twinkv_redundancy(k, synth.WINDOW, ws=ws)
+        elif args.path == "symmetric":
+            out = tk.twinkv_redundancy_symmetric(k, synth.WINDOW, ws=ws)
+        elif args.path == "policy":
             out = tk.twinkv_policy(k, K, threshold=w.tau, out=out, ws=ws)
         elif args.path == "dedup":
             out = tk.twinkv_repair_dedup(k, m, b, threshold=w.tau, want_all=True, out=out, ws=ws)
@@ -298,7 +309,8 @@ def run_ours(args, w, ratio):
 
     if rank != 0:
         return
-    m_total = int(out["nswaps"].clamp(min=0).sum().item()) if "nswaps" in out else 0
+    m_total = (int(out["nswaps"].clamp(min=0).sum().item())
+               if isinstance(out, dict) and "nswaps" in out else 0)
     _report(args, w, ratio, world, U, N, d, ms, prof, e2e_ms, h2d, d2h, chunk, clocks, m_total)
 
 
@@ -360,6 +372,10 @@ def kernel_bytes(path, U, N, d, m_total):
     if path == "policy":
         return {"prep": U * (N * d * 2 + 8 * NP + 16 * N),          # norms, identity layout
                 "repair": U * (4 * N + N)}                             # counts in, mask out
+    if path in ("redundancy", "symmetric"):
+        return {"prep": U * (N * d * 2 + 16 * NP + 16 * N),         # norms, identity layout,
+                                                                       # column scaling
+                "refine": U * N * (2 * d + 28)}                        # k_i, norms, twin, score
     return {"prep": U * (5 * N + N + N * d * 2 + NP * d * 2 + 16 * NP + 16 * N),  # scan, gather,
                                                                                    # column scaling
             "repair": U * (8 * N + N + N) + 8 * m_total,               # b, S0 in; S1 out; swaps
@@ -415,8 +431,11 @@ def _report(args, w, ratio, world, U, N, d, ms, prof, e2e_ms, h2d, d2h, chunk, c
                                    f"{timed_s:.2f} s, seconds long)") if sustained else
                                   (f"{pk_kind} bf16_tflops burst (timed region {timed_s:.2f} s, "
                                    "shorter than the power cap's settling)"),
-                     "kernel": "twk audit_kernel" + (" (count mode)" if args.path == "policy"
-                                                     else ""),
+                     "kernel": "twk audit_kernel" + {"policy": " (count mode)",
+                                                     "symmetric": " (symmetric: upper-triangle "
+                                                                  "tiles; FLOP counted as "
+                                                                  "every tile's)"}.get(
+                                                         args.path, ""),
                      "flops_per_launch": flops,
                      "ms_per_launch": audit_ms_per},
         "kernel_ms_per_step": {k: t / args.steps for k, (n, t) in prof.items()},
@@ -493,10 +512,13 @@ def main():
     ap.add_argument("--e2e-chunk", type=int, default=0,
                     help="units per chunk of the host-buffer call (0: the library default, "
                          "about an eighth of L*H aligned to whole waves of row blocks)")
-    ap.add_argument("--path", choices=("repair", "dedup", "policy"), default="repair",
+    ap.add_argument("--path", choices=("repair", "dedup", "policy", "redundancy", "symmetric"),
+                    default="repair",
                     help="repair: audit + swap (the headline); dedup: the repair that "
                          "never evicts both members of a twin pair; policy: the "
-                         "standalone scorer of Sec. 3.2")
+                         "standalone scorer of Sec. 3.2; redundancy: b_i(all) and twins "
+                         "alone (twinkv_redundancy); symmetric: the same from the "
+                         "upper-triangle tiles (twinkv_redundancy_symmetric)")
     ap.add_argument("--workload", choices=("qwen", "llama", "retrieval", "long"),
                     default="qwen",
                     help="qwen: the Qwen3-4B cache shape the metric is quoted on (the "

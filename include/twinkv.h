@@ -118,7 +118,8 @@ typedef enum {
     TWINKV_OP_REPAIR = 1,
     TWINKV_OP_REPAIR_SELECT = 2,
     TWINKV_OP_POLICY = 3,
-    TWINKV_OP_REPAIR_SELECT_DEDUP = 4
+    TWINKV_OP_REPAIR_SELECT_DEDUP = 4,
+    TWINKV_OP_REDUNDANCY_SYMMETRIC = 5
 } twinkv_op;
 
 /* Kernels, for the profiling hooks. */
@@ -152,6 +153,25 @@ size_t twinkv_workspace_size(twinkv_shape s, int32_t op);
 twinkv_status twinkv_redundancy(const void* keys, twinkv_shape s, int32_t window,
                                 double* out_score, int32_t* out_twin, void* workspace,
                                 size_t workspace_bytes, void* stream);
+
+/*
+ * twinkv_redundancy computed from half the similarity tiles (Sec. 3.5: the audit costs
+ * O(n^2 d) per head; Eq. 1 is symmetric, sim(i,j) = sim(j,i)).  Row block rb (rows
+ * [128 rb, 128 rb + 128)) computes only the 256-column tiles from the one holding
+ * column 128 rb on; each tile's similarities serve both its rows (maxima over its
+ * columns) and its columns (maxima over its rows, the candidates of the rows those
+ * columns stand for).  The two directions meet per row in a packed (value,
+ * position) word combined with atomic maxima: the larger value, the lower position
+ * on a tie, with values that agree to 2^-18 relative counting as tied.  Same
+ * arguments and outputs as twinkv_redundancy; workspace
+ * twinkv_workspace_size(s, TWINKV_OP_REDUNDANCY_SYMMETRIC).  About half the tensor-core
+ * work of twinkv_redundancy, but more work per tile after it (the column maxima are
+ * reduced across the threads that hold the rows).
+ */
+twinkv_status twinkv_redundancy_symmetric(const void* keys, twinkv_shape s, int32_t window,
+                                          double* out_score, int32_t* out_twin,
+                                          void* workspace, size_t workspace_bytes,
+                                          void* stream);
 
 /*
  * Audit of a retained set and the budget-exact repair swap (Sec. 3.4, Eq. 4 and the

@@ -147,7 +147,7 @@ size_t up256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
 struct Layout {
     size_t keys16 = 0, colrinv = 0, colpos = 0, norm2 = 0, ukk = 0, kp = 0, cnt = 0, kb = 0,
            twin0 = 0, twin1 = 0, bret = 0, k0 = 0, i0 = 0, k1 = 0, i1 = 0, rcount = 0,
-           rank = 0;
+           rank = 0, slots = 0;
     size_t total = 0;
 };
 
@@ -162,7 +162,8 @@ Layout layout(const twinkv_shape& s, int op)
     };
     const size_t U = static_cast<size_t>(s.L) * s.H;
     const size_t N = static_cast<size_t>(s.N);
-    if (op == TWINKV_OP_REDUNDANCY || op == TWINKV_OP_REPAIR || op == TWINKV_OP_POLICY) {
+    if (op == TWINKV_OP_REDUNDANCY || op == TWINKV_OP_REPAIR || op == TWINKV_OP_POLICY ||
+        op == TWINKV_OP_REDUNDANCY_SYMMETRIC) {
         const size_t NP = static_cast<size_t>(column_stride(s.N));
         if (s.dtype == TWINKV_F32) L.keys16 = take(U * N * s.d * 2);
         L.colrinv = take(U * NP * 4);
@@ -179,6 +180,7 @@ Layout layout(const twinkv_shape& s, int op)
         }
     }
     if (op == TWINKV_OP_POLICY) L.rcount = take(U * N * 4);
+    if (op == TWINKV_OP_REDUNDANCY_SYMMETRIC) L.slots = take(U * N * 8);
     if (op == TWINKV_OP_REPAIR || op == TWINKV_OP_REPAIR_SELECT ||
         op == TWINKV_OP_REPAIR_SELECT_DEDUP) {
         L.k0 = take(U * N * 8);
@@ -224,7 +226,7 @@ twinkv_status keys_bf16(const void* keys, const twinkv_shape& s, void* ws, const
 
 twinkv_status run_audit(const DeviceInfo& dev, const twinkv_shape& s, const uint16_t* keys16,
                         const void* bkeys, int64_t b_rows, AuditArgs a, cudaStream_t st,
-                        bool count = false)
+                        AuditMode mode = AuditMode::kArgmax)
 {
     CUtensorMap tmA, tmB;
     const int64_t U = static_cast<int64_t>(s.L) * s.H;
@@ -235,7 +237,7 @@ twinkv_status run_audit(const DeviceInfo& dev, const twinkv_shape& s, const uint
     const int64_t items = U * a.RB;
     const int grid = static_cast<int>(items < dev.sms ? items : dev.sms);
     ProfScope p(TWINKV_KERNEL_AUDIT, st);
-    return cuda_status(launch_audit(s.d, count, tmA, tmB, a, grid, st));
+    return cuda_status(launch_audit(s.d, mode, tmA, tmB, a, grid, st));
 }
 
 twinkv_status params_ok(const twinkv_params& p, float threshold)
@@ -452,7 +454,7 @@ size_t twinkv_swaps_capacity(twinkv_shape s)
 
 size_t twinkv_workspace_size(twinkv_shape s, int32_t op)
 {
-    if (op < TWINKV_OP_REDUNDANCY || op > TWINKV_OP_REPAIR_SELECT_DEDUP) return 0;
+    if (op < TWINKV_OP_REDUNDANCY || op > TWINKV_OP_REDUNDANCY_SYMMETRIC) return 0;
     if (!shape_ok(s, op != TWINKV_OP_REPAIR_SELECT && op != TWINKV_OP_REPAIR_SELECT_DEDUP))
         return 0;
     return layout(s, op).total;
@@ -557,14 +559,18 @@ twinkv_status twinkv_profile_end(int32_t* launches, double* total_ms)
     return st;
 }
 
-twinkv_status twinkv_redundancy(const void* keys, twinkv_shape s, int32_t window,
-                                double* out_score, int32_t* out_twin, void* workspace,
-                                size_t workspace_bytes, void* stream)
+}  // extern "C"
+
+namespace {
+twinkv_status redundancy_impl(const void* keys, twinkv_shape s, int32_t window, double* out_score,
+                              int32_t* out_twin, void* workspace, size_t workspace_bytes,
+                              void* stream, bool symmetric)
 {
     if (!keys || !aligned16(keys) || !out_score || !out_twin || window < 0 || !shape_ok(s, true))
         return TWINKV_ERR_INVALID_ARG;
+    const int op = symmetric ? TWINKV_OP_REDUNDANCY_SYMMETRIC : TWINKV_OP_REDUNDANCY;
     Layout L;
-    twinkv_status r = check_ws(s, TWINKV_OP_REDUNDANCY, workspace, workspace_bytes, &L);
+    twinkv_status r = check_ws(s, op, workspace, workspace_bytes, &L);
     if (r != TWINKV_OK) return r;
     DeviceInfo* dev = nullptr;
     if ((r = device_info(&dev)) != TWINKV_OK) return r;
@@ -577,13 +583,16 @@ twinkv_status twinkv_redundancy(const void* keys, twinkv_shape s, int32_t window
     float* colrinv = at<float>(workspace, L.colrinv);
     int* colpos = at<int>(workspace, L.colpos);
     float4* norm2 = at<float4>(workspace, L.norm2);
+    unsigned long long* slots = symmetric ? at<unsigned long long>(workspace, L.slots) : nullptr;
     {
         ProfScope p(TWINKV_KERNEL_PREP, st);
         unsigned* ukk = at<unsigned>(workspace, L.ukk);
         if (cudaMemsetAsync(ukk, 0, static_cast<size_t>(U) * 4, st) != cudaSuccess ||
             launch_norms_identity(k16, U, s.N, s.d, NP, colrinv, colpos, norm2, st, 1.0f, ukk) !=
                 cudaSuccess ||
-            launch_scale_columns(colrinv, U, NP, ukk, st) != cudaSuccess)
+            launch_scale_columns(colrinv, U, NP, ukk, st) != cudaSuccess ||
+            (symmetric && cudaMemsetAsync(slots, 0, static_cast<size_t>(U) * s.N * 8, st) !=
+                              cudaSuccess))
             return TWINKV_ERR_CUDA;
     }
     AuditArgs a;
@@ -599,12 +608,39 @@ twinkv_status twinkv_redundancy(const void* keys, twinkv_shape s, int32_t window
     a.colrinv = colrinv;
     a.colpos = colpos;
     a.out_t0 = out_twin;
+    a.slots = slots;
     a.err = dev->err;
     a.timeout_ns = g_timeout_ns;
     a.mant_mask = 0xFFFFFFE0u;
-    if ((r = run_audit(*dev, s, k16, k16, static_cast<int64_t>(U) * s.N, a, st)) != TWINKV_OK)
+    if ((r = run_audit(*dev, s, k16, k16, static_cast<int64_t>(U) * s.N, a, st,
+                       symmetric ? AuditMode::kSymmetric : AuditMode::kArgmax)) != TWINKV_OK)
         return r;
+    if (symmetric) {
+        ProfScope p(TWINKV_KERNEL_REFINE, st);   // post-processing of the audit's slots
+        if (launch_slots_to_twins(slots, static_cast<int64_t>(U) * s.N, out_twin, st) !=
+            cudaSuccess)
+            return TWINKV_ERR_CUDA;
+    }
     return run_refine(k16, s, norm2, out_twin, nullptr, out_score, nullptr, st);
+}
+}  // namespace
+
+extern "C" {
+
+twinkv_status twinkv_redundancy(const void* keys, twinkv_shape s, int32_t window,
+                                double* out_score, int32_t* out_twin, void* workspace,
+                                size_t workspace_bytes, void* stream)
+{
+    return redundancy_impl(keys, s, window, out_score, out_twin, workspace, workspace_bytes,
+                           stream, false);
+}
+
+twinkv_status twinkv_redundancy_symmetric(const void* keys, twinkv_shape s, int32_t window,
+                                          double* out_score, int32_t* out_twin, void* workspace,
+                                          size_t workspace_bytes, void* stream)
+{
+    return redundancy_impl(keys, s, window, out_score, out_twin, workspace, workspace_bytes,
+                           stream, true);
 }
 
 twinkv_status twinkv_policy(const void* keys, twinkv_shape s, const int32_t* budget,
@@ -655,8 +691,8 @@ twinkv_status twinkv_policy(const void* keys, twinkv_shape s, const int32_t* bud
     a.mant_mask = 0xFFFFFFE0u;
     a.count_tau = threshold;
     a.out_count = count;
-    if ((r = run_audit(*dev, s, k16, k16, static_cast<int64_t>(U) * s.N, a, st, true)) !=
-        TWINKV_OK)
+    if ((r = run_audit(*dev, s, k16, k16, static_cast<int64_t>(U) * s.N, a, st,
+                       AuditMode::kCount)) != TWINKV_OK)
         return r;
     ProfScope pr(TWINKV_KERNEL_REPAIR, st);
     return cuda_status(launch_policy_select(count, U, s.N, budget, p.n_sink, p.n_recent,

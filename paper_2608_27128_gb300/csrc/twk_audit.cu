@@ -60,7 +60,7 @@ constexpr int kGW = kBN / kGroups;            // columns per group (a multiple o
 constexpr int kThreads = 64 + 32 * kEpiWarps; // + TMA warp + MMA warp
 constexpr uint32_t kTmemCols = 512;
 
-template <int D>
+template <int D, bool kSym = false>
 struct AuditCfg {
     static constexpr int KC = D / 64;                 // 128-byte K chunks per key row
     static constexpr int A_CHUNK = kBM * 128;         // 16 KB
@@ -73,8 +73,13 @@ struct AuditCfg {
     static constexpr int OFF_B = OFF_A + 2 * A_BYTES;
     static constexpr int OFF_META = OFF_B + STAGES * B_STAGE;
     static constexpr int OFF_X = OFF_META + MSLOTS * META;   // 2 x (groups-1) x 128 x 16 B
-    static constexpr int OFF_BAR = OFF_X + 2 * (kGroups - 1) * kBM * 16;
-    static constexpr int NBAR = 2 + 2 + 2 * STAGES + 2 * MSLOTS + 2 + 2 + 2 + 2 + 1;
+    // symmetric mode: each group's four warps exchange their per-column maxima here
+    // (two tile parities x groups x 4 lane quarters x 128 columns)
+    static constexpr int OFF_CB = OFF_X + 2 * (kGroups - 1) * kBM * 16;
+    static constexpr int CB_BYTES = kSym ? 2 * kGroups * 4 * kBM * 4 : 0;
+    static constexpr int OFF_BAR = OFF_CB + CB_BYTES;
+    static constexpr int NBAR = 2 + 2 + 2 * STAGES + 2 * MSLOTS + 2 + 2 + 2 + 2 + 1 +
+                                (kSym ? 2 * kGroups : 0);
     static constexpr int OFF_MISC = OFF_BAR + NBAR * 8;
     static constexpr int BYTES = OFF_MISC + 16 + 1024;       // + 1024 for alignment
 };
@@ -265,16 +270,62 @@ __device__ __forceinline__ float count_group(const uint32_t (&x0)[32], const uin
     return c.x + c.y;
 }
 
+__device__ __forceinline__ uint32_t redux_max(uint32_t v)
+{
+    uint32_t r;
+    asm volatile("redux.sync.max.u32 %0, %1, 0xffffffff;" : "=r"(r) : "r"(v));
+    return r;
+}
+
+// Symmetric mode, the column direction of one 32-column chunk: for every column j of
+// the chunk the largest x_ij s_i + kOffset over the warp's 32 rows i (s_i = the row's
+// own column scale, so the value is that of row j's candidate i), its low 5 bits
+// replaced by (31 - lane) so that a tie goes to the lowest row.  Masked: window pairs
+// and rows past the end give 0, below every candidate.  Lane l returns column l's.
+template <bool kMasked>
+__device__ __forceinline__ uint32_t colpass32(const uint32_t (&x)[32], const int* pos, int rw,
+                                              uint32_t w2, float si, bool row_ok)
+{
+    const int lane = threadIdx.x & 31;
+    const uint32_t code = 31u - static_cast<uint32_t>(lane);
+    uint32_t keep = 0u;
+#pragma unroll
+    for (int k = 0; k < 32; k += 4) {
+        int4 q = make_int4(0, 0, 0, 0);
+        if (kMasked) q = *reinterpret_cast<const int4*>(pos + k);
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            float v = fmaf(__uint_as_float(x[k + e]), si, kOffset);
+            if (kMasked) {
+                const int pj = e == 0 ? q.x : e == 1 ? q.y : e == 2 ? q.z : q.w;
+                v = (row_ok && static_cast<uint32_t>(pj - rw) > w2) ? v : 0.f;
+            }
+            const uint32_t r = redux_max((__float_as_uint(v) & 0xFFFFFFE0u) | code);
+            keep = lane == k + e ? r : keep;
+        }
+    }
+    return keep;
+}
+
 struct Tiles {
     int tr;   // tiles of segment 0 (retained, or every column in mode 0)
     int te;   // tiles of segment 1 (evicted; 0 unless b_all is wanted)
+    int t0;   // the first tile (symmetric mode: the tile holding column 128 rb - 0..128)
 };
 
-__device__ __forceinline__ Tiles unit_tiles(const AuditArgs& a, int u)
+// Symmetric mode: row block rb takes the tiles from the one holding its own first
+// column, rb / 2, to the last; the pairs left of them reach rb's rows through the
+// column maxima of the row blocks before it.
+template <bool kSym>
+__device__ __forceinline__ Tiles unit_tiles(const AuditArgs& a, int u, int rb)
 {
-    if (!a.repair_mode) return {(a.N + kBN - 1) / kBN, 0};
+    if (kSym) {
+        const int t0 = rb >> 1;
+        return {(a.N + kBN - 1) / kBN - t0, 0, t0};
+    }
+    if (!a.repair_mode) return {(a.N + kBN - 1) / kBN, 0, 0};
     const int kb = a.kb[u];
-    return {(kb + kBN - 1) / kBN, a.need_all ? (a.N - kb + kBN - 1) / kBN : 0};
+    return {(kb + kBN - 1) / kBN, a.need_all ? (a.N - kb + kBN - 1) / kBN : 0, 0};
 }
 
 // Lane 0 waits, the warp follows its verdict.
@@ -316,12 +367,12 @@ __device__ __forceinline__ int last_parity(long long total, int n, int s)
 
 // Registers are per sub-partition (16384 each): with W warps a sub-partition holds
 // ceil(W / 4) of them, which bounds the registers per thread.
-template <int D, bool kCount>
+template <int D, bool kCount, bool kSym>
 __global__ void __launch_bounds__(kThreads, 1)
     audit_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                  const __grid_constant__ AuditArgs a)
 {
-    using C = AuditCfg<D>;
+    using C = AuditCfg<D, kSym>;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
     uint8_t* sA = smem + C::OFF_A;
@@ -340,6 +391,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint64_t* x_full = t_empty + 2;
     uint64_t* x_empty = x_full + 2;
     uint64_t* drain = x_empty + 2;
+    uint64_t* cbar = drain + 1;   // symmetric mode: [tile parity][group], 128 arrivals
+    uint32_t* sCB = reinterpret_cast<uint32_t*>(smem + C::OFF_CB);
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + C::OFF_MISC);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + C::OFF_MISC + 4);
 
@@ -364,6 +417,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             mbar_init(&m_empty[i], kEpiWarps);
         }
         mbar_init(drain, 1);
+        if (kSym)
+            for (int i = 0; i < 2 * kGroups; ++i) mbar_init(&cbar[i], 4 * 32);
         *abort_flag = 0;
         fence_mbarrier_init();
     }
@@ -391,7 +446,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int item = blockIdx.x; item < n_items && ok; item += gridDim.x) {
             const int u = item / a.RB;
             const int rb = item - u * a.RB;
-            const Tiles ut = unit_tiles(a, u);
+            const Tiles ut = unit_tiles<kSym>(a, u, rb);
             const int ab = static_cast<int>(n_a & 1);
             ok = lane0_wait(&a_empty[ab], static_cast<uint32_t>(((n_a >> 1) & 1) ^ 1), wc, 1);
             if (!ok) break;
@@ -407,7 +462,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             ++n_a;
             const int nt = ut.tr + ut.te;
             for (int t = 0; t < nt && ok; ++t) {
-                const int col0 = t * kBN;
+                const int col0 = (ut.t0 + t) * kBN;
                 const int ms = static_cast<int>(n_m % C::MSLOTS);
                 ok = lane0_wait(&m_empty[ms],
                                 static_cast<uint32_t>(((n_m / C::MSLOTS) & 1) ^ 1), wc, 2);
@@ -459,7 +514,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         bool ok = true;
         for (int item = blockIdx.x; item < n_items && ok; item += gridDim.x) {
             const int u = item / a.RB;
-            const Tiles ut = unit_tiles(a, u);
+            const Tiles ut = unit_tiles<kSym>(a, u, item - u * a.RB);
             const int ab = static_cast<int>(n_a & 1);
             ok = lane0_wait(&a_full[ab], static_cast<uint32_t>((n_a >> 1) & 1), wc, 4);
             if (!ok) break;
@@ -520,14 +575,20 @@ __global__ void __launch_bounds__(kThreads, 1)
         uint32_t ms = 0, mph = 0;    // meta ring slot and phase
         uint32_t acc = 0, tph = 0;   // accumulator buffer and phase
         uint32_t n_x = 0;
+        uint32_t n_c = 0;   // symmetric mode: tiles whose column maxima were merged
         bool ok = true;
         for (int item = blockIdx.x; item < n_items && ok; item += gridDim.x) {
             const int u = item / a.RB;
             const int rb = item - u * a.RB;
-            const Tiles ut = unit_tiles(a, u);
+            const Tiles ut = unit_tiles<kSym>(a, u, rb);
             const int nt = ut.tr + ut.te;
             const int r0 = rb * kBM;
             const int row = r0 + row_local;
+            // symmetric mode: the row's own column scale (the value of row j's candidate
+            // i is x_ij s_i), and whether this row block runs past the end of the unit
+            const bool row_ok = row < a.N;
+            const float si = (kSym && row_ok) ? a.colrinv[static_cast<int64_t>(u) * a.NP + row] : 0.f;
+            const bool pad_item = r0 + kBM > a.N;
 
             // Column ranges that meet the window band [r0 - w, r0 + 128 + w) of this
             // row block: only tiles meeting them need the per-element window test.
@@ -566,7 +627,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const float* rinv = reinterpret_cast<const float*>(sMeta + ms * C::META) + h * kGW;
                 const int* pos =
                     reinterpret_cast<const int*>(sMeta + ms * C::META + kBN * 4) + h * kGW;
-                const int c_lo = t * kBN + h * kGW;
+                const int c_lo = (ut.t0 + t) * kBN + h * kGW;
                 const bool band = (c_lo < s0b && c_lo + kGW > s0a) ||
                                   (c_lo < s1b && c_lo + kGW > s1a);
                 const uint32_t taddr = tmem + lane_base + acc * kBN + static_cast<uint32_t>(h * kGW);
@@ -577,7 +638,67 @@ __global__ void __launch_bounds__(kThreads, 1)
                 tc_fence_before();
                 __syncwarp();
                 if (lane == 0) mbar_arrive(&t_empty[acc]);
-                if (kCount) {
+                if (kSym) {
+                    // row maxima as in mode 0, and each chunk's column maxima over this
+                    // warp's 32 rows right after it (while its registers are live)
+                    uint32_t cr[4];
+                    if (band) {
+                        fold32<true>(x0, rinv, pos, rw, w2, mask, c_lo, b0);
+                        cr[0] = colpass32<true>(x0, pos, rw, w2, si, row_ok);
+                        fold32<true>(x1, rinv + 32, pos + 32, rw, w2, mask, c_lo + 32, b0);
+                        cr[1] = colpass32<true>(x1, pos + 32, rw, w2, si, row_ok);
+                        fold32<true>(x2, rinv + 64, pos + 64, rw, w2, mask, c_lo + 64, b0);
+                        cr[2] = colpass32<true>(x2, pos + 64, rw, w2, si, row_ok);
+                        fold32<true>(x3, rinv + 96, pos + 96, rw, w2, mask, c_lo + 96, b0);
+                        cr[3] = colpass32<true>(x3, pos + 96, rw, w2, si, row_ok);
+                    } else if (pad_item) {
+                        fold32<false>(x0, rinv, pos, rw, w2, mask, c_lo, b0);
+                        cr[0] = colpass32<true>(x0, pos, rw, w2, si, row_ok);
+                        fold32<false>(x1, rinv + 32, pos + 32, rw, w2, mask, c_lo + 32, b0);
+                        cr[1] = colpass32<true>(x1, pos + 32, rw, w2, si, row_ok);
+                        fold32<false>(x2, rinv + 64, pos + 64, rw, w2, mask, c_lo + 64, b0);
+                        cr[2] = colpass32<true>(x2, pos + 64, rw, w2, si, row_ok);
+                        fold32<false>(x3, rinv + 96, pos + 96, rw, w2, mask, c_lo + 96, b0);
+                        cr[3] = colpass32<true>(x3, pos + 96, rw, w2, si, row_ok);
+                    } else {
+                        fold32<false>(x0, rinv, pos, rw, w2, mask, c_lo, b0);
+                        cr[0] = colpass32<false>(x0, pos, rw, w2, si, row_ok);
+                        fold32<false>(x1, rinv + 32, pos + 32, rw, w2, mask, c_lo + 32, b0);
+                        cr[1] = colpass32<false>(x1, pos + 32, rw, w2, si, row_ok);
+                        fold32<false>(x2, rinv + 64, pos + 64, rw, w2, mask, c_lo + 64, b0);
+                        cr[2] = colpass32<false>(x2, pos + 64, rw, w2, si, row_ok);
+                        fold32<false>(x3, rinv + 96, pos + 96, rw, w2, mask, c_lo + 96, b0);
+                        cr[3] = colpass32<false>(x3, pos + 96, rw, w2, si, row_ok);
+                    }
+                    // merge the four lane quarters of this group: the warps exchange their
+                    // 128 column maxima, then warp q takes columns 32q .. 32q + 31
+                    const int par = static_cast<int>(n_c & 1);
+                    uint32_t* cb = sCB + (par * kGroups + h) * 4 * kBM;
+#pragma unroll
+                    for (int k = 0; k < 4; ++k) cb[q * kBM + 32 * k + lane] = cr[k];
+                    mbar_arrive(&cbar[par * kGroups + h]);
+                    ok = all_wait(&cbar[par * kGroups + h], (n_c >> 1) & 1, wc, 11);
+                    ++n_c;
+                    if (!ok) break;
+                    const int c = q * 32 + lane;
+                    uint32_t best = cb[c];
+                    int bq = 0;
+#pragma unroll
+                    for (int qq = 1; qq < 4; ++qq) {
+                        const uint32_t vq = cb[qq * kBM + c];
+                        if ((vq & 0xFFFFFFE0u) > (best & 0xFFFFFFE0u)) {
+                            best = vq;
+                            bq = qq;
+                        }
+                    }
+                    const int gcol = c_lo + c;
+                    if (gcol < a.N && (best & 0xFFFFFFE0u) != 0u) {
+                        const uint32_t win = static_cast<uint32_t>(r0 + 32 * bq + 31) - (best & 31u);
+                        atomicMax(a.slots + static_cast<int64_t>(u) * a.N + gcol,
+                                  (static_cast<unsigned long long>(best & 0xFFFFFFE0u) << 32) |
+                                      (0xFFFFFFFFull - win));
+                    }
+                } else if (kCount) {
                     cnt += band ? count_group<true>(x0, x1, x2, x3, rinv, pos, rw, w2, thr)
                                 : count_group<false>(x0, x1, x2, x3, rinv, pos, rw, w2, thr);
                 } else if (t < ut.tr) {
@@ -646,7 +767,16 @@ __global__ void __launch_bounds__(kThreads, 1)
                     }
                 }
                 mbar_arrive(&x_empty[xb]);
-                if (row < a.N) {
+                if (kSym) {
+                    // the row direction's best joins the column maxima of earlier row
+                    // blocks in the row's slot: value (low 5 bits cleared) then lowest
+                    // position
+                    if (row < a.N && c0 >= 0)
+                        atomicMax(a.slots + static_cast<int64_t>(u) * a.N + row,
+                                  (static_cast<unsigned long long>(__float_as_uint(v0) &
+                                                                   0xFFFFFFE0u) << 32) |
+                                      (0xFFFFFFFFull - static_cast<uint32_t>(c0)));
+                } else if (row < a.N) {
                     const int64_t o_idx = static_cast<int64_t>(u) * a.N + row;
                     const int64_t cbase = static_cast<int64_t>(u) * a.NP;
                     const int p0 = c0 < 0 ? -1 : (a.repair_mode ? a.colpos[cbase + c0] : c0);
@@ -672,26 +802,51 @@ size_t audit_smem_bytes(int d)
     return d == 128 ? AuditCfg<128>::BYTES : AuditCfg<64>::BYTES;
 }
 
-template <int D, bool kCount>
+template <int D, bool kCount, bool kSym>
 cudaError_t launch_audit_t(const CUtensorMap& tmA, const CUtensorMap& tmB, const AuditArgs& a,
                            int grid, cudaStream_t st)
 {
-    const int bytes = AuditCfg<D>::BYTES;
-    cudaError_t e = cudaFuncSetAttribute(audit_kernel<D, kCount>,
+    const int bytes = AuditCfg<D, kSym>::BYTES;
+    cudaError_t e = cudaFuncSetAttribute(audit_kernel<D, kCount, kSym>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
     if (e != cudaSuccess) return e;
-    audit_kernel<D, kCount><<<grid, kThreads, bytes, st>>>(tmA, tmB, a);
+    audit_kernel<D, kCount, kSym><<<grid, kThreads, bytes, st>>>(tmA, tmB, a);
     return cudaGetLastError();
 }
 
-cudaError_t launch_audit(int d, bool count, const CUtensorMap& tmA, const CUtensorMap& tmB,
+cudaError_t launch_audit(int d, AuditMode mode, const CUtensorMap& tmA, const CUtensorMap& tmB,
                          const AuditArgs& a, int grid, cudaStream_t st)
 {
-    if (d == 128)
-        return count ? launch_audit_t<128, true>(tmA, tmB, a, grid, st)
-                     : launch_audit_t<128, false>(tmA, tmB, a, grid, st);
-    return count ? launch_audit_t<64, true>(tmA, tmB, a, grid, st)
-                 : launch_audit_t<64, false>(tmA, tmB, a, grid, st);
+    if (d == 128) {
+        if (mode == AuditMode::kCount) return launch_audit_t<128, true, false>(tmA, tmB, a, grid, st);
+        if (mode == AuditMode::kSymmetric)
+            return launch_audit_t<128, false, true>(tmA, tmB, a, grid, st);
+        return launch_audit_t<128, false, false>(tmA, tmB, a, grid, st);
+    }
+    if (mode == AuditMode::kCount) return launch_audit_t<64, true, false>(tmA, tmB, a, grid, st);
+    if (mode == AuditMode::kSymmetric) return launch_audit_t<64, false, true>(tmA, tmB, a, grid, st);
+    return launch_audit_t<64, false, false>(tmA, tmB, a, grid, st);
+}
+
+namespace {
+// twin of every row from its slot: the low word holds 0xFFFFFFFF - position; an empty
+// slot (no candidate beyond the window) gives -1
+__global__ void slots_to_twins_kernel(const unsigned long long* __restrict__ slots, int64_t n,
+                                      int* __restrict__ twin)
+{
+    const int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+    if (i >= n) return;
+    const unsigned long long sv = slots[i];
+    twin[i] = sv == 0ull ? -1 : static_cast<int>(0xFFFFFFFFull - (sv & 0xFFFFFFFFull));
+}
+}  // namespace
+
+cudaError_t launch_slots_to_twins(const unsigned long long* slots, int64_t n, int* twin,
+                                  cudaStream_t st)
+{
+    const int64_t blocks = (n + 255) / 256;
+    slots_to_twins_kernel<<<static_cast<unsigned>(blocks), 256, 0, st>>>(slots, n, twin);
+    return cudaGetLastError();
 }
 
 // ---------------------------------------------------------------- wait probe

@@ -46,7 +46,13 @@ struct AuditArgs {
     // out_t0/out_t1 unused
     float count_tau;            // tau, compared strictly
     int* out_count;             // [U][N] r_i
+    // symmetric mode (mode 0 columns, upper-triangle tiles): per row, the best
+    // candidate as (value bits with the 5 low bits cleared) << 32 | (0xFFFFFFFF - pos),
+    // combined with atomicMax from both directions; zero-initialised by the caller
+    unsigned long long* slots;  // [U][N]
 };
+
+enum class AuditMode { kArgmax, kCount, kSymmetric };
 
 struct RepairArgs {
     int U, N;
@@ -112,9 +118,13 @@ cudaError_t launch_refine(const uint16_t* keys, int U, int N, int d, const float
 
 // audit kernel (tensor maps built by the caller)
 size_t audit_smem_bytes(int d);
-// count = false: max/argmax (Eq. 1, Eq. 4); true: redundancy counts (Eq. 2)
-cudaError_t launch_audit(int d, bool count, const CUtensorMap& tmA, const CUtensorMap& tmB,
+// kArgmax: max/argmax (Eq. 1, Eq. 4); kCount: redundancy counts (Eq. 2); kSymmetric:
+// max/argmax from the upper-triangle tiles only, into a.slots
+cudaError_t launch_audit(int d, AuditMode mode, const CUtensorMap& tmA, const CUtensorMap& tmB,
                          const AuditArgs& a, int grid, cudaStream_t st);
+// slots [n] (as the symmetric audit leaves them) -> twin positions, -1 for an empty slot
+cudaError_t launch_slots_to_twins(const unsigned long long* slots, int64_t n, int* twin,
+                                  cudaStream_t st);
 
 // standalone policy selection (Sec. 3.2, Eq. 3): per unit, keep budget[u] positions
 // ordered by (protected first, count ascending, position ascending)

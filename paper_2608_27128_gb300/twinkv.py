@@ -23,7 +23,8 @@ from . import build as _build
  ERR_TOO_LARGE) = range(8)
 NOALLOC_MAX_POSITIONS = 262144
 BF16, F32 = 0, 1
-OP_REDUNDANCY, OP_REPAIR, OP_REPAIR_SELECT, OP_POLICY, OP_REPAIR_SELECT_DEDUP = 0, 1, 2, 3, 4
+(OP_REDUNDANCY, OP_REPAIR, OP_REPAIR_SELECT, OP_POLICY, OP_REPAIR_SELECT_DEDUP,
+ OP_REDUNDANCY_SYMMETRIC) = range(6)
 KERNEL_PREP, KERNEL_AUDIT, KERNEL_REPAIR, KERNEL_REFINE = 0, 1, 2, 3
 KERNEL_NAMES = ("prep", "audit", "repair", "refine")
 
@@ -35,6 +36,7 @@ EXPORTED = (
     "twinkv_repair_select_noalloc", "twinkv_host_arena_size", "twinkv_host_default_chunk",
     "twinkv_repair_host",
     "twinkv_policy", "twinkv_repair_dedup", "twinkv_repair_select_dedup",
+    "twinkv_redundancy_symmetric",
 )
 
 
@@ -84,6 +86,7 @@ def load(build_if_missing: bool = True):
         lib.twinkv_workspace_size.restype = ctypes.c_size_t
         lib.twinkv_redundancy.argtypes = [_P, Shape, ctypes.c_int32, _P, _P, _P,
                                           ctypes.c_size_t, _P]
+        lib.twinkv_redundancy_symmetric.argtypes = lib.twinkv_redundancy.argtypes
         lib.twinkv_repair.argtypes = [_P, Shape, _P, _P, ctypes.c_float,
                                       ctypes.POINTER(Params), _P, _P, _P, _P, _P, _P, _P, _P,
                                       _P, ctypes.c_size_t, _P]
@@ -112,7 +115,8 @@ def load(build_if_missing: bool = True):
         lib.twinkv_wait_probe.argtypes = [ctypes.c_uint64, ctypes.POINTER(ctypes.c_int32), _P]
         lib.twinkv_profile_end.argtypes = [ctypes.POINTER(ctypes.c_int32),
                                            ctypes.POINTER(ctypes.c_double)]
-        for name in ("twinkv_redundancy", "twinkv_repair", "twinkv_repair_select",
+        for name in ("twinkv_redundancy", "twinkv_redundancy_symmetric", "twinkv_repair",
+                     "twinkv_repair_select",
                      "twinkv_repair_select_noalloc", "twinkv_repair_host", "twinkv_policy",
                      "twinkv_repair_dedup", "twinkv_repair_select_dedup",
                      "twinkv_get_last_error", "twinkv_set_wait_timeout_ns",
@@ -220,6 +224,23 @@ def twinkv_redundancy(keys, window: int = 32, out_score=None, out_twin=None, ws=
     st = load().twinkv_redundancy(_ptr(keys), s, int(window), _ptr(out_score), _ptr(out_twin),
                                   _ptr(ws), ws.numel(), _stream(stream))
     _check(st, "twinkv_redundancy")
+    return out_score, out_twin
+
+
+def twinkv_redundancy_symmetric(keys, window: int = 32, out_score=None, out_twin=None,
+                                ws=None, stream=None):
+    """twinkv_redundancy from the upper-triangle similarity tiles only (each tile serves
+    its rows and its columns); same arguments and results."""
+    s = shape_of(keys)
+    dev = keys.device
+    _need(keys, "keys", keys.dtype, keys.shape, dev)
+    out_score = _out(out_score, "out_score", torch.float64, keys.shape[:3], dev)
+    out_twin = _out(out_twin, "out_twin", torch.int32, keys.shape[:3], dev)
+    ws = _ws(ws, s, OP_REDUNDANCY_SYMMETRIC, dev)
+    st = load().twinkv_redundancy_symmetric(_ptr(keys), s, int(window), _ptr(out_score),
+                                            _ptr(out_twin), _ptr(ws), ws.numel(),
+                                            _stream(stream))
+    _check(st, "twinkv_redundancy_symmetric")
     return out_score, out_twin
 
 

@@ -24,9 +24,10 @@ def keys_tensor(keys: np.ndarray, L: int, H: int) -> torch.Tensor:
     return t.to(device())
 
 
-def redundancy_vs_oracle(keys, L, H, window, rows=None) -> Report:
+def redundancy_vs_oracle(keys, L, H, window, rows=None, symmetric=False) -> Report:
     U, N, d = keys.shape
-    score, twin = tk.twinkv_redundancy(keys_tensor(keys, L, H), window)
+    call = tk.twinkv_redundancy_symmetric if symmetric else tk.twinkv_redundancy
+    score, twin = call(keys_tensor(keys, L, H), window)
     torch.cuda.synchronize()
     s = score.reshape(U, N).cpu().numpy()
     t = twin.reshape(U, N).cpu().numpy()

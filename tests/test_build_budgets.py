@@ -70,9 +70,17 @@ AUDIT_REGS = 168
 
 @pytest.mark.parametrize("d,count", [(128, 0), (64, 0), (128, 1), (64, 1)])
 def test_audit_kernel_budget(reports, d, count):
-    regs, spill, _ = _one(reports["twk_audit.cu"], rf"audit_kernelILi{d}ELb{count}E")
+    regs, spill, _ = _one(reports["twk_audit.cu"], rf"audit_kernelILi{d}ELb{count}ELb0E")
     assert regs <= AUDIT_REGS
     assert spill <= 8
+
+
+@pytest.mark.parametrize("d", [128, 64])
+def test_symmetric_audit_fits_the_same_launch(reports, d):
+    """The symmetric mode keeps the launch shape (one 320-thread CTA per SM at <= 168
+    registers); its column pass spills, which its measured speed includes."""
+    regs, _, _ = _one(reports["twk_audit.cu"], rf"audit_kernelILi{d}ELb0ELb1E")
+    assert regs <= AUDIT_REGS
 
 
 @pytest.mark.parametrize("d", [128, 64])

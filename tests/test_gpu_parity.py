@@ -126,6 +126,50 @@ def test_redundancy_matches_oracle(L, H, N, d, w):
     assert rep.max_dev_same_twin < 1e-9
 
 
+@pytest.mark.parametrize("L,H,N,d,w", REDUNDANCY_CASES + [(1, 2, 1500, 128, 3), (1, 1, 3000, 64, 32)])
+def test_symmetric_redundancy_matches_oracle(L, H, N, d, w):
+    """The upper-triangle audit: rows meet their earlier candidates through the column
+    maxima of earlier row blocks, in the same packed (value, position) slot."""
+    keys = synth.random_keys(20 + N, L * H, N, d)
+    rep, s, t = redundancy_vs_oracle(keys, L, H, w, symmetric=True)
+    assert rep.n_fail == 0, rep.notes
+    assert rep.n_excused <= max(1, N // 100)
+    assert rep.max_dev_same_twin < 1e-9
+
+
+@pytest.mark.parametrize("n", [64, 128])
+def test_symmetric_exact_ties_go_to_lowest_position(n):
+    """Exact ties through both directions: simplex keys (every similarity -1/(n-1)) and
+    Hadamard rows (every similarity 0), nothing excused."""
+    keys = synth.f32_to_bf16_bits(simplex(n).astype(np.float32))[None]
+    had = synth.f32_to_bf16_bits(hadamard(n).astype(np.float32))[None]
+    i = np.arange(n)
+    for w in (0, 5, 31):
+        for k in (keys, had):
+            score, twin = tk.twinkv_redundancy_symmetric(keys_tensor(k, 1, 1), w)
+            np.testing.assert_array_equal(twin.cpu().numpy().ravel(), np.where(i > w, 0, i + w + 1))
+            rep, s, t = redundancy_vs_oracle(k, 1, 1, w, symmetric=True)
+            assert rep.n_fail == 0 and rep.n_excused == 0, rep.notes
+
+
+def test_symmetric_planted_twins_across_row_blocks():
+    """Planted copies whose source lies in an earlier row block (found only through the
+    column direction) and in a later one (row direction), at several distances."""
+    rng = np.random.default_rng(77)
+    N, d = 2000, 128
+    x = rng.standard_normal((1, N, d)).astype(np.float32)
+    pairs = [(5, 1900), (130, 131 + 200), (700, 260), (1999, 3), (1024, 1500)]
+    for src, dst in pairs:
+        x[0, dst] = x[0, src] + 0.01 * rng.standard_normal(d).astype(np.float32)
+    keys = synth.f32_to_bf16_bits(x)
+    score, twin = tk.twinkv_redundancy_symmetric(keys_tensor(keys, 1, 1), 32)
+    t = twin.cpu().numpy().ravel()
+    for src, dst in pairs:
+        assert t[dst] == src and t[src] == dst
+    rep, s, tt = redundancy_vs_oracle(keys, 1, 1, 32, symmetric=True)
+    assert rep.n_fail == 0, rep.notes
+
+
 REPAIR_CASES = [
     # L, H, N, d, w, K, tau, n_sink, n_recent
     (1, 1, 1, 64, 0, 1, 0.85, 4, 64),

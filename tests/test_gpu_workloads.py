@@ -198,3 +198,37 @@ def test_redundancy_full_size_many_items_per_cta(name):
            planted_excused=0, max_dev_same_twin=rep.max_dev_same_twin)
     assert rep.n_fail == 0, rep.notes
     assert rep.max_dev_same_twin < 1e-9
+
+
+def test_symmetric_redundancy_full_qwen_shape():
+    """twinkv_redundancy_symmetric at the full Qwen3-4B shape (36 x 8 x 16384 x 128):
+    128 random rows of every unit against the oracle, every planted twin exact, and the
+    twins equal to the full-tile audit's wherever that one is not a near tie."""
+    w = synth.get("qwen")
+    keys, truths = synth.keys(w)
+    U, N = w.units, w.N
+    kt = keys_tensor(keys, w.L, w.H)
+    score, twin = tk.twinkv_redundancy_symmetric(kt, synth.WINDOW)
+    torch.cuda.synchronize()
+    assert tk.twinkv_get_last_error() == tk.OK
+    s = score.reshape(U, N).cpu().numpy()
+    t = twin.reshape(U, N).cpu().numpy()
+    del kt, score, twin
+    torch.cuda.empty_cache()
+    rng = np.random.default_rng(23)
+    rep = Report()
+    n_rows = 0
+    for u in range(U):
+        rows = np.sort(rng.choice(N, size=128, replace=False))
+        a = oracle.audit(keys[u:u + 1], window=synth.WINDOW, rows=rows)
+        sim = (lambda uu: (lambda i, j: oracle.sim(keys, uu, i, j)))(u)
+        rep.add(compare_best(s[u, rows], t[u, rows], a["b_all"][0], a["t_all"][0],
+                             a["b_all2"][0], sim, synth.WINDOW, rows=rows, what=f"u{u}"))
+        n_rows += rows.size
+    n_planted = planted(truths, {"twin_all": t}, None)
+    record(workload="qwen", call="twinkv_redundancy_symmetric", units=U, N=N, d=w.d,
+           rows_sampled=n_rows, n_fail=rep.n_fail, excused_twin_all=rep.n_excused,
+           planted_checked=n_planted, planted_excused=0,
+           max_dev_same_twin=rep.max_dev_same_twin)
+    assert rep.n_fail == 0, rep.notes
+    assert rep.max_dev_same_twin < 1e-9
