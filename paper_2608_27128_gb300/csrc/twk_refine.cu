@@ -22,17 +22,45 @@
 namespace twk {
 namespace {
 
-// sim(i, j) of Eq. 1 from the dot product and the two keys' norm records.
-__device__ __forceinline__ double cosine(DF dot, float4 ni, float4 nj)
+// This GPU's FP64 pipe runs at a small fraction of its FP32 rate, so the values stay
+// double-floats until each output is written: comparisons are made on the pairs, and a
+// pair becomes a double by widening both floats with integer operations and one fp64
+// addition (exact: the pair's 48 significant bits fit in a double).
+
+// A float as a double, for zero and normal floats by moving its bits (the conversion
+// instruction for the rest, which similarity values do not reach).
+__device__ __forceinline__ double widen(float f)
 {
-    if (ni.x == 0.f || nj.x == 0.f) return 0.0;   // a zero key has similarity 0
+    const uint32_t u = __float_as_uint(f);
+    const uint32_t e = (u >> 23) & 0xFFu;
+    const uint64_t sign = static_cast<uint64_t>(u & 0x80000000u) << 32;
+    if ((u & 0x7FFFFFFFu) == 0u) return __longlong_as_double(static_cast<long long>(sign));
+    if (e == 0u || e == 0xFFu) return static_cast<double>(f);
+    return __longlong_as_double(static_cast<long long>(
+        sign | (static_cast<uint64_t>(e + 896u) << 52) | (static_cast<uint64_t>(u & 0x7FFFFFu) << 29)));
+}
+
+__device__ __forceinline__ double to_double(DF a) { return widen(a.h) + widen(a.l); }
+
+// a > b and a == b for normalised pairs (|l| at most half an ulp of h).
+__device__ __forceinline__ bool df_gt(DF a, DF b) { return a.h > b.h || (a.h == b.h && a.l > b.l); }
+__device__ __forceinline__ bool df_eq(DF a, DF b) { return a.h == b.h && a.l == b.l; }
+
+// sim(i, j) of Eq. 1 from the dot product and the two keys' norm records, as a
+// double-float.
+__device__ __forceinline__ DF cosine(DF dot, float4 ni, float4 nj)
+{
+    if (ni.x == 0.f || nj.x == 0.f) return DF{0.f, 0.f};   // a zero key has similarity 0
     const DF c = df_mul(dot, df_mul(DF{ni.z, ni.w}, DF{nj.z, nj.w}));
-    if (fabsf(c.h) < 1.0f - 0x1p-20f) return df_to_double(c);
+    if (fabsf(c.h) < 1.0f - 0x1p-20f) return c;
     // Within 2^-20 of +-1: the exact fp64 form, which gives exactly +-1 when the keys
-    // are parallel (a duplicate, or a copy scaled by a power of two).
-    const double si = df_to_double(DF{ni.x, ni.y});
-    const double sj = df_to_double(DF{nj.x, nj.y});
-    return df_to_double(dot) / sqrt(si * sj);
+    // are parallel (a duplicate, or a copy scaled by a power of two), split back into a
+    // pair (its leading 48 bits).
+    const double si = to_double(DF{ni.x, ni.y});
+    const double sj = to_double(DF{nj.x, nj.y});
+    const double x = to_double(dot) / sqrt(si * sj);
+    const float h = static_cast<float>(x);
+    return DF{h, static_cast<float>(x - static_cast<double>(h))};
 }
 
 constexpr int kRefineThreads = 256;
@@ -70,17 +98,18 @@ __global__ void __launch_bounds__(kRefineThreads, kMinBlocks)
     else
         d0 = group_dot_df<D>(ki, keys + s0 * D, part);
     // lane 0 of the group evaluates the first cosine, lane 1 the second
-    double v = -1.0;
+    DF v{-1.f, 0.f};
     if (part == 0 && j0 >= 0) v = cosine(d0, norms[r], norms[s0]);
     if (part == 1 && j1 >= 0) v = cosine(d1, norms[r], norms[s1]);
-    const double v0 = v;
-    const double v1 = __shfl_down_sync(0xFFFFFFFFu, v, 1);
+    const DF v0 = v;
+    const DF v1{__shfl_down_sync(0xFFFFFFFFu, v.h, 1), __shfl_down_sync(0xFFFFFFFFu, v.l, 1)};
     if (part == 0 && live) {
-        b0[r] = v0;
+        b0[r] = to_double(v0);
         if (twin1) {
-            const bool take1 = j1 >= 0 && (j0 < 0 || v1 > v0 || (v1 == v0 && j1 < j0));
+            const bool take1 =
+                j1 >= 0 && (j0 < 0 || df_gt(v1, v0) || (df_eq(v1, v0) && j1 < j0));
             twin1[r] = take1 ? j1 : j0;
-            if (b1) b1[r] = take1 ? v1 : v0;
+            if (b1) b1[r] = to_double(take1 ? v1 : v0);
         }
     }
 }

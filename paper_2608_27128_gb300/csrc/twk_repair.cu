@@ -38,10 +38,19 @@ namespace {
 constexpr int kT = 512;   // two blocks per SM: every unit of a prefill in one wave
 constexpr int kW = kT / 32;
 
+// Order-preserving map of an fp64 value to a u64 key (-0 folded into +0), in integer
+// operations only: fp64 comparisons run on this GPU's narrow FP64 pipe.
 __device__ __forceinline__ uint64_t ordered(double b)
 {
-    const uint64_t u = static_cast<uint64_t>(__double_as_longlong(b == 0.0 ? 0.0 : b));
+    uint64_t u = static_cast<uint64_t>(__double_as_longlong(b));
+    if (u == 0x8000000000000000ull) u = 0ull;
     return (u >> 63) ? ~u : (u | 0x8000000000000000ull);
+}
+
+__device__ __forceinline__ bool is_nan_bits(double b)
+{
+    return (static_cast<uint64_t>(__double_as_longlong(b)) & 0x7FFFFFFFFFFFFFFFull) >
+           0x7FF0000000000000ull;
 }
 
 struct Shared {
@@ -540,7 +549,7 @@ __global__ void __launch_bounds__(kT, 2) select_kernel(const RepairArgs a)
     int* I1 = a.idx1 + off;
     const int S = slice_len(N, C);
     const int lo = min(N, r * S), hi = min(N, lo + S);
-    const double tau = a.tau;
+    const uint64_t ktau = ordered(a.tau);
 
     // A. S1 = S0, counts, and the slice's lists (orphans forward from lo, donors
     // backward from hi: donor k in position order sits at hi - 1 - k).  A thread takes
@@ -583,16 +592,20 @@ __global__ void __launch_bounds__(kT, 2) select_kernel(const RepairArgs a)
                 }
             }
         }
+        // b < tau and b >= tau decided on the order-preserving keys (a NaN b is
+        // neither an orphan nor a donor, as in fp64 comparisons)
         int fo[kEA], fd[kEA], co = 0, cd = 0;
+        uint64_t kv[kEA];
 #pragma unroll
         for (int j = 0; j < kEA; ++j) {
             const int i = i0 + j;
-            const bool in = i < hi;
+            const bool in = i < hi && !is_nan_bits(bv[j]);
+            kv[j] = ordered(bv[j]);
             bad |= mv[j] > 1u;
             cnt += mv[j] != 0u;
             const bool prot = i < a.n_sink || i >= N - a.n_recent;
-            fo[j] = in && mv[j] == 0u && bv[j] < tau;
-            fd[j] = in && mv[j] != 0u && !prot && bv[j] >= tau;
+            fo[j] = in && mv[j] == 0u && kv[j] < ktau;
+            fd[j] = in && mv[j] != 0u && !prot && kv[j] >= ktau;
             co += fo[j];
             cd += fd[j];
         }
@@ -602,12 +615,12 @@ __global__ void __launch_bounds__(kT, 2) select_kernel(const RepairArgs a)
         for (int j = 0; j < kEA; ++j) {
             const int i = i0 + j;
             if (fo[j]) {
-                K0[lo + my_o + po] = ordered(bv[j]);
+                K0[lo + my_o + po] = kv[j];
                 I0[lo + my_o + po] = i;
                 ++po;
             }
             if (fd[j]) {
-                K0[hi - 1 - (my_d + pd)] = ~ordered(bv[j]);
+                K0[hi - 1 - (my_d + pd)] = ~kv[j];
                 I0[hi - 1 - (my_d + pd)] = i;
                 ++pd;
             }
@@ -876,7 +889,9 @@ __global__ void __launch_bounds__(kT, 2) dedup_kernel(const RepairArgs a)   // 2
 
     // 1. validation, counts, and S1 = S0 (also the answer for a failed unit or m = 0)
     int bad = 0, cnt = 0, no = 0, nd = 0;
-    const double tau = a.tau;
+    // b < tau and b >= tau decided on the order-preserving keys (integer operations;
+    // a NaN b is neither an orphan nor a donor, as in fp64 comparisons)
+    const uint64_t ktau = ordered(a.tau);
     for (int c0 = 0; c0 < N; c0 += kT * kE) {
 #pragma unroll
         for (int j = 0; j < kE; ++j) {
@@ -884,12 +899,14 @@ __global__ void __launch_bounds__(kT, 2) dedup_kernel(const RepairArgs a)   // 2
             if (i < N) {
                 const uint8_t v = S0[i];
                 const double bi = b[i];
+                const uint64_t ki = ordered(bi);
+                const bool num = !is_nan_bits(bi);
                 S1[i] = v;
                 bad |= v > 1;
                 cnt += v != 0;
                 const bool prot = i < a.n_sink || i >= N - a.n_recent;
-                no += (v == 0 && bi < tau);
-                nd += (v != 0 && !prot && bi >= tau);
+                no += (v == 0 && num && ki < ktau);
+                nd += (v != 0 && !prot && num && ki >= ktau);
             }
         }
     }
@@ -938,8 +955,10 @@ __global__ void __launch_bounds__(kT, 2) dedup_kernel(const RepairArgs a)   // 2
                 const uint8_t v = S0[i];
                 bv[j] = b[i];
                 const bool prot = i < a.n_sink || i >= N - a.n_recent;
-                fo[j] = (v == 0 && bv[j] < tau);
-                fd[j] = (v != 0 && !prot && bv[j] >= tau);
+                const uint64_t kj = ordered(bv[j]);
+                const bool num = !is_nan_bits(bv[j]);
+                fo[j] = (v == 0 && num && kj < ktau);
+                fd[j] = (v != 0 && !prot && num && kj >= ktau);
             }
             co += fo[j];
             cd += fd[j];
