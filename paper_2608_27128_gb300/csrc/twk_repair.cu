@@ -513,6 +513,53 @@ __device__ __forceinline__ int count_before(const uint64_t* sk, const int* si, i
     return pos;
 }
 
+constexpr int kR = 8;   // items per thread in the share sort's registers
+
+// Compare-exchange of two items: afterwards a orders before b when `up`, after it
+// otherwise.
+__device__ __forceinline__ void cx(uint64_t& ka, int& pa, uint64_t& kb, int& pb, bool up)
+{
+    const bool sw = before(kb, pb, ka, pa) == up;
+    const uint64_t k0 = sw ? kb : ka, k1 = sw ? ka : kb;
+    const int p0 = sw ? pb : pa, p1 = sw ? pa : pb;
+    ka = k0;
+    kb = k1;
+    pa = p0;
+    pb = p1;
+}
+
+// kR items between registers and the shared-memory slots [at, at + kR) (16-byte
+// aligned: at is a multiple of kR).
+__device__ __forceinline__ void store_run(uint64_t* sk, int* si, int at, const uint64_t* kx,
+                                          const int* px)
+{
+#pragma unroll
+    for (int e = 0; e < kR; e += 2)
+        *reinterpret_cast<ulonglong2*>(sk + at + e) = make_ulonglong2(kx[e], kx[e + 1]);
+#pragma unroll
+    for (int e = 0; e < kR; e += 4)
+        *reinterpret_cast<int4*>(si + at + e) = make_int4(px[e], px[e + 1], px[e + 2], px[e + 3]);
+}
+
+__device__ __forceinline__ void load_run(const uint64_t* sk, const int* si, int at, uint64_t* kx,
+                                         int* px)
+{
+#pragma unroll
+    for (int e = 0; e < kR; e += 2) {
+        const ulonglong2 v = *reinterpret_cast<const ulonglong2*>(sk + at + e);
+        kx[e] = v.x;
+        kx[e + 1] = v.y;
+    }
+#pragma unroll
+    for (int e = 0; e < kR; e += 4) {
+        const int4 v = *reinterpret_cast<const int4*>(si + at + e);
+        px[e] = v.x;
+        px[e + 1] = v.y;
+        px[e + 2] = v.z;
+        px[e + 3] = v.w;
+    }
+}
+
 constexpr int kEA = 8;   // consecutive positions per thread in the classification pass
 
 // Slice length: ceil(N / C) rounded up to a multiple of kEA.
@@ -802,39 +849,78 @@ __global__ void __launch_bounds__(kT, 2) select_kernel(const RepairArgs a)
     // C. the swap list: m items per side in severity order
     const int q = (m + C - 1) / C;
     if (q <= kChunk) {
-        int P = 1;
+        // Each CTA sorts its share of both lists by (key, position) with a bitonic
+        // network over P = 2^k >= max(q, kR) slots per side; padding sorts last.  Thread
+        // tt of a side holds the slots [kR*tt, kR*tt + kR) in registers: strides below
+        // kR are exchanged inside the thread, strides up to 16*kR between the lanes of
+        // a warp by shuffles, and longer ones through shared memory.
+        int P = kR;
         while (P < q) P <<= 1;
+        const int TP = P / kR;   // threads per side; threads from 2*TP on hold padding
+        const int side = tid >= TP;
+        const int tt = tid - side * TP;
+        const bool live = tid < 2 * TP;
         const int c_lo = min(m, r * q), c_n = min(m, c_lo + q) - c_lo;
-        for (int t = tid; t < P; t += kT) {
-            const bool in = t < c_n;
-            sk_o[t] = in ? K1[c_lo + t] : ~0ull;
-            si_o[t] = in ? I1[c_lo + t] : 0x7FFFFFFF;
-            sk_d[t] = in ? K1[half + c_lo + t] : ~0ull;
-            si_d[t] = in ? I1[half + c_lo + t] : 0x7FFFFFFF;
+        uint64_t* sk = side ? sk_d : sk_o;
+        int* si = side ? si_d : si_o;
+        uint64_t kx[kR];
+        int px[kR];
+#pragma unroll
+        for (int e = 0; e < kR; ++e) {
+            const int t = tt * kR + e;
+            const bool in = live && t < c_n;
+            kx[e] = in ? K1[side * half + c_lo + t] : ~0ull;
+            px[e] = in ? I1[side * half + c_lo + t] : 0x7FFFFFFF;
         }
-        __syncthreads();
         for (int size = 2; size <= P; size <<= 1) {
-            for (int stride = size >> 1; stride > 0; stride >>= 1) {
-                for (int t = tid; t < P; t += kT) {   // t < P/2: orphans, else donors
-                    const int side = t >= P / 2;
-                    const int tt = side ? t - P / 2 : t;
-                    uint64_t* sk = side ? sk_d : sk_o;
-                    int* si = side ? si_d : si_o;
-                    const int lo2 = 2 * tt - (tt & (stride - 1));
-                    const int hi2 = lo2 + stride;
-                    const uint64_t ka = sk[lo2], kb = sk[hi2];
-                    const int pa = si[lo2], pb = si[hi2];
-                    const bool gt = ka > kb || (ka == kb && pa > pb);
-                    if (gt == ((lo2 & size) == 0)) {
-                        sk[lo2] = kb;
-                        sk[hi2] = ka;
-                        si[lo2] = pb;
-                        si[hi2] = pa;
+            const bool up_t = ((tt * kR) & size) == 0;   // the direction once size >= kR
+            if (size >= 64 * kR) {
+                if (live) store_run(sk, si, tt * kR, kx, px);
+                __syncthreads();
+                for (int stride = size >> 1; stride >= 32 * kR; stride >>= 1) {
+                    for (int t = tid; t < P; t += kT) {   // t < P/2: orphans, else donors
+                        const int sd = t >= P / 2;
+                        const int ts = sd ? t - P / 2 : t;
+                        uint64_t* k2 = sd ? sk_d : sk_o;
+                        int* i2 = sd ? si_d : si_o;
+                        const int lo2 = 2 * ts - (ts & (stride - 1));
+                        const int hi2 = lo2 + stride;
+                        uint64_t ka = k2[lo2], kb = k2[hi2];
+                        int pa = i2[lo2], pb = i2[hi2];
+                        cx(ka, pa, kb, pb, (lo2 & size) == 0);
+                        k2[lo2] = ka;
+                        k2[hi2] = kb;
+                        i2[lo2] = pa;
+                        i2[hi2] = pb;
+                    }
+                    __syncthreads();
+                }
+                if (live) load_run(sk, si, tt * kR, kx, px);
+            }
+            for (int stride = min(size >> 1, 16 * kR); stride >= kR; stride >>= 1) {
+                const int lm = stride / kR;
+                const bool keep_first = ((tt & lm) == 0) == up_t;
+#pragma unroll
+                for (int e = 0; e < kR; ++e) {
+                    const uint64_t ok = __shfl_xor_sync(0xFFFFFFFFu, kx[e], lm);
+                    const int op = __shfl_xor_sync(0xFFFFFFFFu, px[e], lm);
+                    if (before(ok, op, kx[e], px[e]) == keep_first) {
+                        kx[e] = ok;
+                        px[e] = op;
                     }
                 }
-                __syncthreads();
+            }
+#pragma unroll
+            for (int stride = kR / 2; stride > 0; stride >>= 1) {
+                if (stride >= size) continue;
+#pragma unroll
+                for (int e = 0; e < kR; ++e)
+                    if ((e & stride) == 0)
+                        cx(kx[e], px[e], kx[e + stride], px[e + stride],
+                           (((tt * kR) | e) & size) == 0);
             }
         }
+        if (live) store_run(sk, si, tt * kR, kx, px);
         cluster_sync<C>();   // every share is sorted
         for (int t = tid; t < 2 * c_n; t += kT) {
             const int side = t >= c_n;
