@@ -92,6 +92,15 @@ __global__ void __launch_bounds__(kRefineThreads, kMinBlocks)
     // stood in for by the row itself and its value discarded.
     const int64_t s0 = base + (j0 >= 0 ? j0 : r - base);
     const int64_t s1 = base + (j1 >= 0 ? j1 : r - base);
+    // The standalone launch loads the norm records the cosine needs (the row's, and
+    // the twin's this lane evaluates) beside the keys rather than after the dot
+    // product; the launch beside the audit has no registers to hold them.
+    constexpr bool kEarly = kMinBlocks < 6;
+    float4 nr{}, nt{};
+    if constexpr (kEarly) {
+        nr = norms[r];
+        nt = norms[part == 1 ? s1 : s0];
+    }
     DF d0, d1{0.f, 0.f};
     if (__any_sync(0xFFFFFFFFu, j1 >= 0))   // both dots at once, one per f32x2 half
         group_dot2_df<D>(ki, keys + s0 * D, keys + s1 * D, part, d0, d1);
@@ -99,8 +108,8 @@ __global__ void __launch_bounds__(kRefineThreads, kMinBlocks)
         d0 = group_dot_df<D>(ki, keys + s0 * D, part);
     // lane 0 of the group evaluates the first cosine, lane 1 the second
     DF v{-1.f, 0.f};
-    if (part == 0 && j0 >= 0) v = cosine(d0, norms[r], norms[s0]);
-    if (part == 1 && j1 >= 0) v = cosine(d1, norms[r], norms[s1]);
+    if (part == 0 && j0 >= 0) v = cosine(d0, kEarly ? nr : norms[r], kEarly ? nt : norms[s0]);
+    if (part == 1 && j1 >= 0) v = cosine(d1, kEarly ? nr : norms[r], kEarly ? nt : norms[s1]);
     const DF v0 = v;
     const DF v1{__shfl_down_sync(0xFFFFFFFFu, v.h, 1), __shfl_down_sync(0xFFFFFFFFu, v.l, 1)};
     if (part == 0 && live) {

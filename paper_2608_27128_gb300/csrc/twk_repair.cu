@@ -750,6 +750,7 @@ __global__ void __launch_bounds__(kT, 2) select_kernel(const RepairArgs a)
         int need = m;
         bool whole = false;
         int pass = 0;
+        int below = 0, at_cut = 0;   // this CTA's items below the cut and at it, per digit
         for (int shift = 56; shift >= 0 && !whole; shift -= 8, ++pass) {
             int* h = cs.hist[pass & 1];
             if (tid < 256) h[tid] = 0;
@@ -772,10 +773,12 @@ __global__ void __launch_bounds__(kT, 2) select_kernel(const RepairArgs a)
                 }
             }
             cluster_sync<C>();   // every CTA's histogram of this pass is complete
+            int own = 0;
             if (tid < 256) {
                 int t = 0;
                 for (int q = 0; q < C; ++q) t += peer<C>(h, q)[tid];
                 s.base[tid] = t;
+                own = h[tid];
             }
             __syncthreads();
             if (tid < 32) digit_cut(s.base, need, s.sel_digit, s.sel_before, s.sel_count);
@@ -784,16 +787,14 @@ __global__ void __launch_bounds__(kT, 2) select_kernel(const RepairArgs a)
             prefix |= static_cast<uint64_t>(s.sel_digit) << shift;
             pmask |= 255ull << shift;
             whole = s.sel_count == need;
+            // digit tid of this CTA's own histogram: below the selected digit, or at it
+            below += tid < s.sel_digit ? own : 0;
+            at_cut = tid == s.sel_digit ? own : 0;
             __syncthreads();
         }
         // ordered compaction: every item below the cut (and at it when `whole`), then
         // the first `need` items at the cut in position order over the cluster
-        int nl = 0, ne = 0;
-        for (int k = tid; k < mine; k += kT) {
-            const uint64_t km = item_key(x, k) & pmask;
-            nl += km < prefix || (whole && km == prefix);
-            ne += !whole && km == prefix;
-        }
+        int nl = below + (whole ? at_cut : 0), ne = whole ? 0 : at_cut;
         if (tid < 2) s.red[tid] = 0;
         __syncthreads();
         nl = __reduce_add_sync(0xFFFFFFFFu, nl);
@@ -820,25 +821,38 @@ __global__ void __launch_bounds__(kT, 2) select_kernel(const RepairArgs a)
         }
         __syncthreads();
         int base = cs.tot[6], seen_eq = cs.tot[7];
-        for (int c0 = 0; c0 < mine; c0 += kT) {
-            const int k = c0 + tid;
-            int fl = 0, fe = 0;
-            uint64_t key = 0;
-            int pos = 0;
-            if (k < mine) {
-                key = item_key(x, k);
-                pos = item_pos(x, k);
-                const uint64_t km = key & pmask;
-                fl = km < prefix || (whole && km == prefix);
-                fe = !whole && km == prefix;
+        for (int c0 = 0; c0 < mine; c0 += kT * kEA) {
+            // a thread takes kEA consecutive items; fl: below the cut (or at it when
+            // `whole`), fe: at the cut
+            const int k0 = c0 + tid * kEA;
+            uint64_t kk[kEA];
+            int pp[kEA];
+            uint32_t fl = 0, fe = 0;
+#pragma unroll
+            for (int j = 0; j < kEA; ++j) {
+                kk[j] = 0;
+                pp[j] = 0;
+                if (k0 + j < mine) {
+                    kk[j] = item_key(x, k0 + j);
+                    pp[j] = item_pos(x, k0 + j);
+                    const uint64_t km = kk[j] & pmask;
+                    fl |= static_cast<uint32_t>(km < prefix || (whole && km == prefix)) << j;
+                    fe |= static_cast<uint32_t>(!whole && km == prefix) << j;
+                }
             }
             int pl, pe, tl, te;
-            scan2(s, fl, fe, pl, pe, tl, te);
+            scan2n(s, __popc(fl), __popc(fe), pl, pe, tl, te);
             const int k_eq = max(0, min(te, need - seen_eq));   // taken at the cut here
-            if (fl || (fe && pe < k_eq)) {
-                const int dst = base + pl + min(pe, k_eq);
-                K1[dst0 + dst] = key;
-                I1[dst0 + dst] = pos;
+#pragma unroll
+            for (int j = 0; j < kEA; ++j) {
+                const int l = (fl >> j) & 1, e = (fe >> j) & 1;
+                if (l || (e && pe < k_eq)) {
+                    const int dst = base + pl + min(pe, k_eq);
+                    K1[dst0 + dst] = kk[j];
+                    I1[dst0 + dst] = pp[j];
+                }
+                pl += l;
+                pe += e;
             }
             base += tl + k_eq;
             seen_eq += te;
