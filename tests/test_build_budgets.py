@@ -94,7 +94,10 @@ def test_refine_beside_an_audit_cta_fits(reports, d):
 @pytest.mark.parametrize("d", [128, 64])
 def test_standalone_refine_budget(reports, d):
     regs, spill, _ = _one(reports["twk_refine.cu"], rf"refine_kernelILi{d}ELi5E")
-    assert regs <= 48 and spill == 0
+    # Five blocks per SM.  Loading the norm records beside the keys costs ptxas a few
+    # bytes of spill at this cap (4 with nvcc 13.0) and still measured faster
+    # than the spill-free order (0.535 against 0.578 ms at the Qwen3-4B shape).
+    assert regs <= 48 and spill <= 8
 
 
 def test_dedup_repair_two_blocks_per_sm(reports):
