@@ -862,98 +862,107 @@ __global__ void __launch_bounds__(kT, 2) select_kernel(const RepairArgs a)
 
     // C. the swap list: m items per side in severity order
     const int q = (m + C - 1) / C;
-    if (q <= kChunk) {
+    if (q <= 2 * kChunk) {
         // Each CTA sorts its share of both lists by (key, position) with a bitonic
         // network over P = 2^k >= max(q, kR) slots per side; padding sorts last.  Thread
         // tt of a side holds the slots [kR*tt, kR*tt + kR) in registers: strides below
         // kR are exchanged inside the thread, strides up to 16*kR between the lanes of
-        // a warp by shuffles, and longer ones through shared memory.
+        // a warp by shuffles, and longer ones through shared memory.  Shares of up to
+        // kChunk items sort both sides at once (half of the threads and of the buffer
+        // each); longer ones (up to 2*kChunk) sort one side after the other, each over
+        // all threads and the whole buffer (sk_o..sk_d and si_o..si_d are contiguous).
+        const bool both = q <= kChunk;
+        const int nside = both ? 2 : 1;
         int P = kR;
         while (P < q) P <<= 1;
-        const int TP = P / kR;   // threads per side; threads from 2*TP on hold padding
-        const int side = tid >= TP;
-        const int tt = tid - side * TP;
-        const bool live = tid < 2 * TP;
+        const int TP = P / kR;   // threads per side; threads from nside*TP on hold padding
         const int c_lo = min(m, r * q), c_n = min(m, c_lo + q) - c_lo;
-        uint64_t* sk = side ? sk_d : sk_o;
-        int* si = side ? si_d : si_o;
-        uint64_t kx[kR];
-        int px[kR];
+        for (int pass = 0; pass < 3 - nside; ++pass) {
+            const int sd = both && tid >= TP;     // the thread's side among those sorted
+            const int side = both ? sd : pass;    // 0: orphans, 1: donors
+            const int tt = tid - sd * TP;
+            const bool live = tid < nside * TP;
+            uint64_t* sk = sd ? sk_d : sk_o;
+            int* si = sd ? si_d : si_o;
+            uint64_t kx[kR];
+            int px[kR];
 #pragma unroll
-        for (int e = 0; e < kR; ++e) {
-            const int t = tt * kR + e;
-            const bool in = live && t < c_n;
-            kx[e] = in ? K1[side * half + c_lo + t] : ~0ull;
-            px[e] = in ? I1[side * half + c_lo + t] : 0x7FFFFFFF;
-        }
-        for (int size = 2; size <= P; size <<= 1) {
-            const bool up_t = ((tt * kR) & size) == 0;   // the direction once size >= kR
-            if (size >= 64 * kR) {
-                if (live) store_run(sk, si, tt * kR, kx, px);
-                __syncthreads();
-                for (int stride = size >> 1; stride >= 32 * kR; stride >>= 1) {
-                    for (int t = tid; t < P; t += kT) {   // t < P/2: orphans, else donors
-                        const int sd = t >= P / 2;
-                        const int ts = sd ? t - P / 2 : t;
-                        uint64_t* k2 = sd ? sk_d : sk_o;
-                        int* i2 = sd ? si_d : si_o;
-                        const int lo2 = 2 * ts - (ts & (stride - 1));
-                        const int hi2 = lo2 + stride;
-                        uint64_t ka = k2[lo2], kb = k2[hi2];
-                        int pa = i2[lo2], pb = i2[hi2];
-                        cx(ka, pa, kb, pb, (lo2 & size) == 0);
-                        k2[lo2] = ka;
-                        k2[hi2] = kb;
-                        i2[lo2] = pa;
-                        i2[hi2] = pb;
-                    }
+            for (int e = 0; e < kR; ++e) {
+                const int t = tt * kR + e;
+                const bool in = live && t < c_n;
+                kx[e] = in ? K1[side * half + c_lo + t] : ~0ull;
+                px[e] = in ? I1[side * half + c_lo + t] : 0x7FFFFFFF;
+            }
+            for (int size = 2; size <= P; size <<= 1) {
+                const bool up_t = ((tt * kR) & size) == 0;   // the direction once size >= kR
+                if (size >= 64 * kR) {
+                    if (live) store_run(sk, si, tt * kR, kx, px);
                     __syncthreads();
+                    for (int stride = size >> 1; stride >= 32 * kR; stride >>= 1) {
+                        for (int t = tid; t < nside * (P / 2); t += kT) {
+                            const int s2 = t >= P / 2;   // pairs of the second side (both)
+                            const int ts = s2 ? t - P / 2 : t;
+                            uint64_t* k2 = s2 ? sk_d : sk_o;
+                            int* i2 = s2 ? si_d : si_o;
+                            const int lo2 = 2 * ts - (ts & (stride - 1));
+                            const int hi2 = lo2 + stride;
+                            uint64_t ka = k2[lo2], kb = k2[hi2];
+                            int pa = i2[lo2], pb = i2[hi2];
+                            cx(ka, pa, kb, pb, (lo2 & size) == 0);
+                            k2[lo2] = ka;
+                            k2[hi2] = kb;
+                            i2[lo2] = pa;
+                            i2[hi2] = pb;
+                        }
+                        __syncthreads();
+                    }
+                    if (live) load_run(sk, si, tt * kR, kx, px);
                 }
-                if (live) load_run(sk, si, tt * kR, kx, px);
-            }
-            for (int stride = min(size >> 1, 16 * kR); stride >= kR; stride >>= 1) {
-                const int lm = stride / kR;
-                const bool keep_first = ((tt & lm) == 0) == up_t;
+                for (int stride = min(size >> 1, 16 * kR); stride >= kR; stride >>= 1) {
+                    const int lm = stride / kR;
+                    const bool keep_first = ((tt & lm) == 0) == up_t;
 #pragma unroll
-                for (int e = 0; e < kR; ++e) {
-                    const uint64_t ok = __shfl_xor_sync(0xFFFFFFFFu, kx[e], lm);
-                    const int op = __shfl_xor_sync(0xFFFFFFFFu, px[e], lm);
-                    if (before(ok, op, kx[e], px[e]) == keep_first) {
-                        kx[e] = ok;
-                        px[e] = op;
+                    for (int e = 0; e < kR; ++e) {
+                        const uint64_t ok = __shfl_xor_sync(0xFFFFFFFFu, kx[e], lm);
+                        const int op = __shfl_xor_sync(0xFFFFFFFFu, px[e], lm);
+                        if (before(ok, op, kx[e], px[e]) == keep_first) {
+                            kx[e] = ok;
+                            px[e] = op;
+                        }
                     }
                 }
-            }
 #pragma unroll
-            for (int stride = kR / 2; stride > 0; stride >>= 1) {
-                if (stride >= size) continue;
+                for (int stride = kR / 2; stride > 0; stride >>= 1) {
+                    if (stride >= size) continue;
 #pragma unroll
-                for (int e = 0; e < kR; ++e)
-                    if ((e & stride) == 0)
-                        cx(kx[e], px[e], kx[e + stride], px[e + stride],
-                           (((tt * kR) | e) & size) == 0);
+                    for (int e = 0; e < kR; ++e)
+                        if ((e & stride) == 0)
+                            cx(kx[e], px[e], kx[e + stride], px[e + stride],
+                               (((tt * kR) | e) & size) == 0);
+                }
             }
+            if (live) store_run(sk, si, tt * kR, kx, px);
+            cluster_sync<C>();   // every share of the sides sorted in this pass is sorted
+            for (int t = tid; t < nside * c_n; t += kT) {
+                const int s2 = t >= c_n;
+                const int ts = s2 ? t - c_n : t;
+                const int sdx = both ? s2 : pass;   // 0: orphans, 1: donors
+                const uint64_t* k2 = s2 ? sk_d : sk_o;
+                const int* i2 = s2 ? si_d : si_o;
+                const uint64_t key = k2[ts];
+                const int pos = i2[ts];
+                // its rank: its place in its own share plus, in every other share, the
+                // number of items ordered before it
+                int rank = ts;
+                for (int qq = 0; qq < C; ++qq)
+                    if (qq != r)
+                        rank += count_before(peer<C>(const_cast<uint64_t*>(k2), qq),
+                                             peer<C>(const_cast<int*>(i2), qq), P, key, pos);
+                swaps[2 * rank + (sdx ? 0 : 1)] = pos;
+                S1[pos] = sdx ? 0 : 1;
+            }
+            cluster_sync<C>();   // every lookup into this CTA's shares is done
         }
-        if (live) store_run(sk, si, tt * kR, kx, px);
-        cluster_sync<C>();   // every share is sorted
-        for (int t = tid; t < 2 * c_n; t += kT) {
-            const int side = t >= c_n;
-            const int tt = side ? t - c_n : t;
-            const uint64_t* sk = side ? sk_d : sk_o;
-            const int* si = side ? si_d : si_o;
-            const uint64_t key = sk[tt];
-            const int pos = si[tt];
-            // its rank: its place in its own share plus, in every other share, the
-            // number of items ordered before it
-            int rank = tt;
-            for (int qq = 0; qq < C; ++qq)
-                if (qq != r)
-                    rank += count_before(peer<C>(const_cast<uint64_t*>(sk), qq),
-                                         peer<C>(const_cast<int*>(si), qq), P, key, pos);
-            swaps[2 * rank + (side ? 0 : 1)] = pos;
-            S1[pos] = side ? 0 : 1;
-        }
-        cluster_sync<C>();   // every lookup into this CTA's shares is done
     } else {
         // long lists: one CTA per side sorts its m items with the stable radix passes
         // (keys0/idx0, free by now, as the second buffer)

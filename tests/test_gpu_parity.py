@@ -313,9 +313,9 @@ def test_repair_select_is_bit_exact(seed):
 
 @pytest.mark.parametrize("N,frac", [(30000, 0.5), (24001, 0.35)])
 def test_repair_select_lists_on_both_sides_of_the_shared_memory_sort(N, frac):
-    """Lists of the m selected items up to 4096 are sorted in shared memory, longer ones
-    by radix passes: units with m well above and well below 4096, many equal b values
-    and ties at tau, bit-exact against the oracle's selection."""
+    """Units whose swap lists run from a few dozen items to well above 4096, at the
+    cluster size the library picks for them, with many equal b values and ties at tau,
+    bit-exact against the oracle's selection."""
     rng = np.random.default_rng(N)
     L, H = 1, 4
     U = L * H
@@ -342,9 +342,10 @@ def test_repair_select_lists_on_both_sides_of_the_shared_memory_sort(N, frac):
                                      (50, 25, 0.0)])
 def test_repair_select_every_cluster_size(cluster, N, K, tau, monkeypatch):
     """The literal selection on clusters of 1 to 16 CTAs per unit (forced; the library
-    picks the size from the unit count): lists cut on either side, shares of the swap
-    list above and below the per-CTA shared-memory sort (2048 items), slices that are
-    empty, many equal b values and ties at tau, bit-exact against the oracle."""
+    picks the size from the unit count): lists cut on either side; per-CTA shares of the
+    swap list up to 2048 items (both sides sorted at once), from 2049 to 4096 (one side
+    after the other) and above (radix passes over the workspace); slices that are empty,
+    many equal b values and ties at tau, bit-exact against the oracle."""
     monkeypatch.setenv("TWINKV_SELECT_CLUSTER", str(cluster))
     rng = np.random.default_rng([N, K, cluster])
     L, H = 1, 3
