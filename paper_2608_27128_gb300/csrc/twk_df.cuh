@@ -1,7 +1,7 @@
 // twk_df.cuh -- double-float arithmetic (an unevaluated sum of two floats) and the one
 // dot-product routine behind every exact similarity value of the TwinKV pass: bf16 x
 // bf16 products are exact in fp32 and are accumulated with Knuth's TwoSum, four lanes
-// per dot product, each over a contiguous quarter, combined in a fixed tree.  Every
+// per dot product, each over every fourth 16-byte chunk, combined in a fixed tree.  Every
 // dot product (norms included) goes through group_dot_df, so identical keys give
 // identical values and the value of k_i . k_j equals that of k_j . k_i bit for bit.
 #pragma once
@@ -36,23 +36,25 @@ __device__ __forceinline__ void df_add(float& hi, float& lo, float hi2, float lo
     lo = __fsub_rn(e, __fsub_rn(hi, s));
 }
 
-constexpr int kParts = 4;   // threads per dot product, each over a contiguous quarter
+constexpr int kParts = 4;   // threads per dot product, each over every fourth 16-byte chunk
 
-// One quarter of a . b for two bf16 rows of length D: terms in increasing t.
+// One lane's part of a . b for two bf16 rows of length D: the 16-byte chunks part,
+// part + kParts, part + 2 kParts, ... (so that the kParts lanes of a dot product read
+// kParts * 16 contiguous bytes per load), terms in increasing t.
 template <int D>
 __device__ __forceinline__ void quarter_dot(const uint16_t* __restrict__ a,
                                             const uint16_t* __restrict__ b, int part,
                                             float& hi, float& lo)
 {
-    constexpr int Q = D / 8 / kParts;   // 16-byte chunks per quarter
-    const uint4* a4 = reinterpret_cast<const uint4*>(a) + part * Q;
-    const uint4* b4 = reinterpret_cast<const uint4*>(b) + part * Q;
+    constexpr int Q = D / 8 / kParts;   // 16-byte chunks per lane
+    const uint4* a4 = reinterpret_cast<const uint4*>(a) + part;
+    const uint4* b4 = reinterpret_cast<const uint4*>(b) + part;
     hi = 0.f;
     lo = 0.f;
 #pragma unroll
     for (int q = 0; q < Q; ++q) {
-        const uint4 va = __ldg(a4 + q);
-        const uint4 vb = __ldg(b4 + q);
+        const uint4 va = __ldg(a4 + q * kParts);
+        const uint4 vb = __ldg(b4 + q * kParts);
         const uint32_t wa[4] = {va.x, va.y, va.z, va.w};
         const uint32_t wb[4] = {vb.x, vb.y, vb.z, vb.w};
 #pragma unroll
@@ -66,7 +68,7 @@ __device__ __forceinline__ void quarter_dot(const uint16_t* __restrict__ a,
 }
 
 // a . b by the kParts consecutive lanes of a group (every lane passes its part): the
-// quarters are summed as ((q0 + q1) + (q2 + q3)), and every lane of the group returns
+// lanes' parts are summed as ((q0 + q1) + (q2 + q3)), and every lane of the group returns
 // the same double-float.  All dot products, norms included, go through this routine.
 template <int D>
 __device__ __forceinline__ DFPair group_dot_df(const uint16_t* __restrict__ a,
@@ -109,22 +111,23 @@ __device__ __forceinline__ void df_add2(float2& hi, float2& lo, float2 hi2, floa
     lo = __fadd2_rn(e, neg2(__fadd2_rn(hi, neg2(s))));
 }
 
+// b1 is read only where use1 (elsewhere its terms are zero and r1 is meaningless).
 template <int D>
 __device__ __forceinline__ void group_dot2_df(const uint16_t* __restrict__ a,
                                               const uint16_t* __restrict__ b0,
-                                              const uint16_t* __restrict__ b1, int part,
-                                              DFPair& r0, DFPair& r1)
+                                              const uint16_t* __restrict__ b1, bool use1,
+                                              int part, DFPair& r0, DFPair& r1)
 {
     constexpr int Q = D / 8 / kParts;
-    const uint4* a4 = reinterpret_cast<const uint4*>(a) + part * Q;
-    const uint4* c4 = reinterpret_cast<const uint4*>(b0) + part * Q;
-    const uint4* d4 = reinterpret_cast<const uint4*>(b1) + part * Q;
+    const uint4* a4 = reinterpret_cast<const uint4*>(a) + part;
+    const uint4* c4 = reinterpret_cast<const uint4*>(b0) + part;
+    const uint4* d4 = reinterpret_cast<const uint4*>(b1) + part;
     float2 hi = make_float2(0.f, 0.f), lo = make_float2(0.f, 0.f);
 #pragma unroll
     for (int q = 0; q < Q; ++q) {
-        const uint4 va = __ldg(a4 + q);
-        const uint4 vc = __ldg(c4 + q);
-        const uint4 vd = __ldg(d4 + q);
+        const uint4 va = __ldg(a4 + q * kParts);
+        const uint4 vc = __ldg(c4 + q * kParts);
+        const uint4 vd = use1 ? __ldg(d4 + q * kParts) : make_uint4(0u, 0u, 0u, 0u);
         const uint32_t wa[4] = {va.x, va.y, va.z, va.w};
         const uint32_t wc[4] = {vc.x, vc.y, vc.z, vc.w};
         const uint32_t wd[4] = {vd.x, vd.y, vd.z, vd.w};

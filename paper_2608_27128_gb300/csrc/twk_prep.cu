@@ -156,10 +156,12 @@ __global__ void __launch_bounds__(kPrepThreads)
         const int r = p - N;
         col = r < kpad - k ? k + r : kpad + (N - k) + (r - (kpad - k));
     }
-    const uint4* src = reinterpret_cast<const uint4*>(key) + part * Q;
-    uint4* dst = reinterpret_cast<uint4*>(kp + (u * NP + col) * D) + part * Q;
+    // the lane's 16-byte chunks part, part + kParts, ... (those its dot product read)
+    const uint4* src = reinterpret_cast<const uint4*>(key) + part;
+    uint4* dst = reinterpret_cast<uint4*>(kp + (u * NP + col) * D) + part;
 #pragma unroll
-    for (int q = 0; q < Q; ++q) dst[q] = p < N ? __ldg(src + q) : make_uint4(0u, 0u, 0u, 0u);
+    for (int q = 0; q < Q; ++q)
+        dst[q * kParts] = p < N ? __ldg(src + q * kParts) : make_uint4(0u, 0u, 0u, 0u);
     if (part == 0) {
         colrinv[u * NP + col] = p < N ? r32 : nan_f();
         colpos[u * NP + col] = p < N ? p : -1;

@@ -8,7 +8,7 @@
 // with every dot product formed as a double-float sum: each bf16 x bf16 product is
 // exact in fp32, and the running sum is an unevaluated pair (hi, lo) updated with
 // Knuth's TwoSum, so its error is of order 2^-48 of the sum of |products|.  Four lanes
-// share a dot product (a contiguous quarter each, combined in a fixed tree).  The
+// share a dot product (every fourth 16-byte chunk each, combined in a fixed tree).  The
 // cosine is then (k_i . k_j) * (1/||k_i|| * 1/||k_j||) in double-float arithmetic
 // (relative error below 1e-12; fp64 square roots and quotients are slow on this GPU),
 // except within 2^-20 of +-1, where the exact fp64 form is used.  All dot products
@@ -103,7 +103,7 @@ __global__ void __launch_bounds__(kRefineThreads, kMinBlocks)
     }
     DF d0, d1{0.f, 0.f};
     if (__any_sync(0xFFFFFFFFu, j1 >= 0))   // both dots at once, one per f32x2 half
-        group_dot2_df<D>(ki, keys + s0 * D, keys + s1 * D, part, d0, d1);
+        group_dot2_df<D>(ki, keys + s0 * D, keys + s1 * D, j1 >= 0, part, d0, d1);
     else
         d0 = group_dot_df<D>(ki, keys + s0 * D, part);
     // lane 0 of the group evaluates the first cosine, lane 1 the second
