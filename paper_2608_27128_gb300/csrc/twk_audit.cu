@@ -151,7 +151,7 @@ constexpr float kOffset = 1.0f + 0x1p-10f;
 // The values are positive, where a larger low-bit code means a larger float, so ties
 // go to the lowest column whatever the sign of the similarity.  Most chunks cost one
 // fused multiply-add and one max tree.
-template <bool kMasked>
+template <bool kMasked, bool kEager = false>
 __device__ __forceinline__ void fold32(const uint32_t (&x)[32], const float* rinv,
                                        const int* pos, int rw, uint32_t w2, uint32_t mask,
                                        int col0, Best& b)
@@ -178,6 +178,22 @@ __device__ __forceinline__ void fold32(const uint32_t (&x)[32], const float* rin
             v[k + 2] = (static_cast<uint32_t>(q.z - rw) > w2) ? v[k + 2] : nan_f();
             v[k + 3] = (static_cast<uint32_t>(q.w - rw) > w2) ? v[k + 3] : nan_f();
         }
+    }
+    if constexpr (kEager) {
+        // Early in a row block some row of the warp improves in most chunks, and the
+        // vote only adds a branch: every value is packed, one tree gives the lowest
+        // column among the values equal to the maximum at 2^-18 relative, and the
+        // running best moves at that resolution (an earlier column keeps a tie).
+        float p[32];
+#pragma unroll
+        for (int k = 0; k < 32; ++k) p[k] = pack(v[k], 31u - static_cast<uint32_t>(k), mask);
+        const uint32_t mp = __float_as_uint(tree32(p));
+        const float m = __uint_as_float(mp & mask);
+        if (m > b.v) {
+            b.v = m;
+            b.col = col0 + 31 - static_cast<int>(mp & 31u);
+        }
+        return;
     }
     const float m = tree32(v);
     const bool up = m > b.v;
@@ -211,16 +227,39 @@ __device__ __forceinline__ void load_group(uint32_t taddr, uint32_t (&x0)[32], u
 }
 
 // Folds the loaded group into the running best, 32 columns at a time in column order.
-template <bool kMasked>
+template <bool kMasked, bool kEager>
 __device__ __forceinline__ void reduce_group(const uint32_t (&x0)[32], const uint32_t (&x1)[32],
                                              const uint32_t (&x2)[32], const uint32_t (&x3)[32],
                                              const float* rinv, const int* pos, int rw,
                                              uint32_t w2, uint32_t mask, int col0, Best& b)
 {
-    fold32<kMasked>(x0, rinv, pos, rw, w2, mask, col0, b);
-    fold32<kMasked>(x1, rinv + 32, pos + 32, rw, w2, mask, col0 + 32, b);
-    fold32<kMasked>(x2, rinv + 64, pos + 64, rw, w2, mask, col0 + 64, b);
-    fold32<kMasked>(x3, rinv + 96, pos + 96, rw, w2, mask, col0 + 96, b);
+    fold32<kMasked, kEager>(x0, rinv, pos, rw, w2, mask, col0, b);
+    fold32<kMasked, kEager>(x1, rinv + 32, pos + 32, rw, w2, mask, col0 + 32, b);
+    fold32<kMasked, kEager>(x2, rinv + 64, pos + 64, rw, w2, mask, col0 + 64, b);
+    fold32<kMasked, kEager>(x3, rinv + 96, pos + 96, rw, w2, mask, col0 + 96, b);
+}
+
+// Folds one tile's group, eagerly (every chunk resolved, no vote) or vote-gated.
+template <bool kEager>
+__device__ __forceinline__ void reduce_tile(bool band, const uint32_t (&x0)[32],
+                                            const uint32_t (&x1)[32], const uint32_t (&x2)[32],
+                                            const uint32_t (&x3)[32], const float* rinv,
+                                            const int* pos, int rw, uint32_t w2, uint32_t mask,
+                                            int col0, Best& b)
+{
+    if (band) reduce_group<true, kEager>(x0, x1, x2, x3, rinv, pos, rw, w2, mask, col0, b);
+    else reduce_group<false, kEager>(x0, x1, x2, x3, rinv, pos, rw, w2, mask, col0, b);
+}
+
+// The tiles of a row block folded eagerly: at d = 64 every tile (a tile's epilogue is
+// twice the tensor-core time there, and with fewer columns per row the running best
+// improves in most chunks); at d = 128 the first 16 tiles of the row block, where some
+// row of a warp improves in most chunks (measured: 16 beat 8 and 32 at the Qwen3-4B
+// shape).
+template <int D>
+__device__ __forceinline__ constexpr int eager_tiles()
+{
+    return D == 64 ? (1 << 30) : 16;
 }
 
 // sat(a * b + c): fp32 fused multiply-add clamped to [0, 1], NaN to 0.
@@ -702,8 +741,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                     cnt += band ? count_group<true>(x0, x1, x2, x3, rinv, pos, rw, w2, thr)
                                 : count_group<false>(x0, x1, x2, x3, rinv, pos, rw, w2, thr);
                 } else if (t < ut.tr) {
-                    if (band) reduce_group<true>(x0, x1, x2, x3, rinv, pos, rw, w2, mask, c_lo, b0);
-                    else reduce_group<false>(x0, x1, x2, x3, rinv, pos, rw, w2, mask, c_lo, b0);
+                    if (t < eager_tiles<D>())
+                        reduce_tile<true>(band, x0, x1, x2, x3, rinv, pos, rw, w2, mask, c_lo, b0);
+                    else
+                        reduce_tile<false>(band, x0, x1, x2, x3, rinv, pos, rw, w2, mask, c_lo, b0);
                 } else {
                     if (t == ut.tr) {
                         // The evicted segment matters only where it reaches the retained
@@ -712,8 +753,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                         // FLT_MIN keeps an exact tie at 0 in play).
                         b1.v = b0.v - (fabsf(b0.v) * 0x1p-13f + FLT_MIN);
                     }
-                    if (band) reduce_group<true>(x0, x1, x2, x3, rinv, pos, rw, w2, mask, c_lo, b1);
-                    else reduce_group<false>(x0, x1, x2, x3, rinv, pos, rw, w2, mask, c_lo, b1);
+                    // the evicted segment: eager at d = 64 only
+                    reduce_tile<D == 64>(band, x0, x1, x2, x3, rinv, pos, rw, w2, mask, c_lo, b1);
                 }
                 __syncwarp();
                 if (lane == 0) mbar_arrive(&m_empty[ms]);

@@ -3,7 +3,7 @@ from ptxas's resource report (-Xptxas -v) of an sm_103a compile of the sources. 
 GPU is needed.
 
 - The audit kernel runs one 320-thread CTA per SM at <= 168 registers (10 warps, three
-  per scheduler) without spilling in its hot loop.
+  per scheduler), with at most a few bytes of spill.
 - The refine instantiation that runs beside an audit CTA (twinkv_repair_host) must fit
   in the registers that CTA leaves free: 168 x 320 + r x 256 <= 65536.
 - The standalone refine keeps its 48-register budget.
@@ -72,7 +72,11 @@ AUDIT_REGS = 168
 def test_audit_kernel_budget(reports, d, count):
     regs, spill, _ = _one(reports["twk_audit.cu"], rf"audit_kernelILi{d}ELb{count}ELb0E")
     assert regs <= AUDIT_REGS
-    assert spill <= 8
+    # The argmax mode carries two fold forms (eager on the first tiles of a row block,
+    # vote-gated after them); with both, ptxas spills 20 bytes at d = 128 and 12 at
+    # d = 64 (nvcc 13.0), and the kernel still measured faster than with the
+    # vote-gated form alone (4 bytes).
+    assert spill <= (24 if count == 0 else 8)
 
 
 @pytest.mark.parametrize("d", [128, 64])
