@@ -678,35 +678,36 @@ __global__ void __launch_bounds__(kThreads, 1)
                 __syncwarp();
                 if (lane == 0) mbar_arrive(&t_empty[acc]);
                 if (kSym) {
-                    // row maxima as in mode 0, and each chunk's column maxima over this
-                    // warp's 32 rows right after it (while its registers are live)
+                    // row maxima (the eager fold: the column pass already costs more than
+                    // the vote saves) and each chunk's column maxima over this warp's 32
+                    // rows right after it (while its registers are live)
                     uint32_t cr[4];
                     if (band) {
-                        fold32<true>(x0, rinv, pos, rw, w2, mask, c_lo, b0);
+                        fold32<true, true>(x0, rinv, pos, rw, w2, mask, c_lo, b0);
                         cr[0] = colpass32<true>(x0, pos, rw, w2, si, row_ok);
-                        fold32<true>(x1, rinv + 32, pos + 32, rw, w2, mask, c_lo + 32, b0);
+                        fold32<true, true>(x1, rinv + 32, pos + 32, rw, w2, mask, c_lo + 32, b0);
                         cr[1] = colpass32<true>(x1, pos + 32, rw, w2, si, row_ok);
-                        fold32<true>(x2, rinv + 64, pos + 64, rw, w2, mask, c_lo + 64, b0);
+                        fold32<true, true>(x2, rinv + 64, pos + 64, rw, w2, mask, c_lo + 64, b0);
                         cr[2] = colpass32<true>(x2, pos + 64, rw, w2, si, row_ok);
-                        fold32<true>(x3, rinv + 96, pos + 96, rw, w2, mask, c_lo + 96, b0);
+                        fold32<true, true>(x3, rinv + 96, pos + 96, rw, w2, mask, c_lo + 96, b0);
                         cr[3] = colpass32<true>(x3, pos + 96, rw, w2, si, row_ok);
                     } else if (pad_item) {
-                        fold32<false>(x0, rinv, pos, rw, w2, mask, c_lo, b0);
+                        fold32<false, true>(x0, rinv, pos, rw, w2, mask, c_lo, b0);
                         cr[0] = colpass32<true>(x0, pos, rw, w2, si, row_ok);
-                        fold32<false>(x1, rinv + 32, pos + 32, rw, w2, mask, c_lo + 32, b0);
+                        fold32<false, true>(x1, rinv + 32, pos + 32, rw, w2, mask, c_lo + 32, b0);
                         cr[1] = colpass32<true>(x1, pos + 32, rw, w2, si, row_ok);
-                        fold32<false>(x2, rinv + 64, pos + 64, rw, w2, mask, c_lo + 64, b0);
+                        fold32<false, true>(x2, rinv + 64, pos + 64, rw, w2, mask, c_lo + 64, b0);
                         cr[2] = colpass32<true>(x2, pos + 64, rw, w2, si, row_ok);
-                        fold32<false>(x3, rinv + 96, pos + 96, rw, w2, mask, c_lo + 96, b0);
+                        fold32<false, true>(x3, rinv + 96, pos + 96, rw, w2, mask, c_lo + 96, b0);
                         cr[3] = colpass32<true>(x3, pos + 96, rw, w2, si, row_ok);
                     } else {
-                        fold32<false>(x0, rinv, pos, rw, w2, mask, c_lo, b0);
+                        fold32<false, true>(x0, rinv, pos, rw, w2, mask, c_lo, b0);
                         cr[0] = colpass32<false>(x0, pos, rw, w2, si, row_ok);
-                        fold32<false>(x1, rinv + 32, pos + 32, rw, w2, mask, c_lo + 32, b0);
+                        fold32<false, true>(x1, rinv + 32, pos + 32, rw, w2, mask, c_lo + 32, b0);
                         cr[1] = colpass32<false>(x1, pos + 32, rw, w2, si, row_ok);
-                        fold32<false>(x2, rinv + 64, pos + 64, rw, w2, mask, c_lo + 64, b0);
+                        fold32<false, true>(x2, rinv + 64, pos + 64, rw, w2, mask, c_lo + 64, b0);
                         cr[2] = colpass32<false>(x2, pos + 64, rw, w2, si, row_ok);
-                        fold32<false>(x3, rinv + 96, pos + 96, rw, w2, mask, c_lo + 96, b0);
+                        fold32<false, true>(x3, rinv + 96, pos + 96, rw, w2, mask, c_lo + 96, b0);
                         cr[3] = colpass32<false>(x3, pos + 96, rw, w2, si, row_ok);
                     }
                     // merge the four lane quarters of this group: the warps exchange their
