@@ -180,10 +180,10 @@ __device__ __forceinline__ void fold32(const uint32_t (&x)[32], const float* rin
         }
     }
     if constexpr (kEager) {
-        // Early in a row block some row of the warp improves in most chunks, and the
-        // vote only adds a branch: every value is packed, one tree gives the lowest
-        // column among the values equal to the maximum at 2^-18 relative, and the
-        // running best moves at that resolution (an earlier column keeps a tie).
+        // Where some row of the warp improves in most chunks the vote only adds a
+        // branch: every value is packed, one tree gives the lowest column among the
+        // values equal to the maximum at 2^-18 relative, and the running best moves at
+        // that resolution (an earlier column keeps a tie).
         float p[32];
 #pragma unroll
         for (int k = 0; k < 32; ++k) p[k] = pack(v[k], 31u - static_cast<uint32_t>(k), mask);
@@ -251,15 +251,17 @@ __device__ __forceinline__ void reduce_tile(bool band, const uint32_t (&x0)[32],
     else reduce_group<false, kEager>(x0, x1, x2, x3, rinv, pos, rw, w2, mask, col0, b);
 }
 
-// The tiles of a row block folded eagerly: at d = 64 every tile (a tile's epilogue is
-// twice the tensor-core time there, and with fewer columns per row the running best
-// improves in most chunks); at d = 128 the first 16 tiles of the row block, where some
-// row of a warp improves in most chunks (measured: 16 beat 8 and 32 at the Qwen3-4B
-// shape).
+// The argmax modes fold eagerly at d = 64 only.  There a tile's epilogue is twice its
+// tensor-core time and, with fewer columns per row, the running best improves in most
+// chunks: the eager fold measured 661 TFLOP/s against 617 at the Llama-3.2-1B shape.  It
+// compares candidates of different chunks at the packed resolution, so more near ties
+// (within 2^-18 relative of the maximum) go to the earlier column; at d = 128 it gained
+// nothing measurable (16 eager tiles per row block: 1275 against 1271 TFLOP/s), and the
+// vote-gated fold keeps the exact comparison across chunks there.
 template <int D>
-__device__ __forceinline__ constexpr int eager_tiles()
+__device__ __forceinline__ constexpr bool eager_fold()
 {
-    return D == 64 ? (1 << 30) : 16;
+    return D == 64;
 }
 
 // sat(a * b + c): fp32 fused multiply-add clamped to [0, 1], NaN to 0.
@@ -742,10 +744,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                     cnt += band ? count_group<true>(x0, x1, x2, x3, rinv, pos, rw, w2, thr)
                                 : count_group<false>(x0, x1, x2, x3, rinv, pos, rw, w2, thr);
                 } else if (t < ut.tr) {
-                    if (t < eager_tiles<D>())
-                        reduce_tile<true>(band, x0, x1, x2, x3, rinv, pos, rw, w2, mask, c_lo, b0);
-                    else
-                        reduce_tile<false>(band, x0, x1, x2, x3, rinv, pos, rw, w2, mask, c_lo, b0);
+                    reduce_tile<eager_fold<D>()>(band, x0, x1, x2, x3, rinv, pos, rw, w2, mask,
+                                                 c_lo, b0);
                 } else {
                     if (t == ut.tr) {
                         // The evicted segment matters only where it reaches the retained
@@ -754,8 +754,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                         // FLT_MIN keeps an exact tie at 0 in play).
                         b1.v = b0.v - (fabsf(b0.v) * 0x1p-13f + FLT_MIN);
                     }
-                    // the evicted segment: eager at d = 64 only
-                    reduce_tile<D == 64>(band, x0, x1, x2, x3, rinv, pos, rw, w2, mask, c_lo, b1);
+                    reduce_tile<eager_fold<D>()>(band, x0, x1, x2, x3, rinv, pos, rw, w2, mask,
+                                                 c_lo, b1);
                 }
                 __syncwarp();
                 if (lane == 0) mbar_arrive(&m_empty[ms]);

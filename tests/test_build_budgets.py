@@ -72,11 +72,10 @@ AUDIT_REGS = 168
 def test_audit_kernel_budget(reports, d, count):
     regs, spill, _ = _one(reports["twk_audit.cu"], rf"audit_kernelILi{d}ELb{count}ELb0E")
     assert regs <= AUDIT_REGS
-    # The argmax mode carries two fold forms (eager on the first tiles of a row block,
-    # vote-gated after them); with both, ptxas spills 20 bytes at d = 128 and 12 at
-    # d = 64 (nvcc 13.0), and the kernel still measured faster than with the
-    # vote-gated form alone (4 bytes).
-    assert spill <= (24 if count == 0 else 8)
+    # At d = 64 the argmax mode folds eagerly (no warp vote); ptxas spills 12 bytes
+    # there (nvcc 13.0), and the kernel still measured faster than with the vote-gated
+    # fold (4 bytes).
+    assert spill <= (16 if (count == 0 and d == 64) else 8)
 
 
 @pytest.mark.parametrize("d", [128, 64])
