@@ -460,19 +460,22 @@ __host__ __device__ inline size_t dedup_kernel_smem_bytes(int N)
 //      m = min(|O|, |D|).  The side with more than m items is cut by a radix select
 //      whose digit histograms are summed over the cluster (each CTA histograms its own
 //      items; the sums, and so every decision, are identical in every CTA); the other
-//      side is taken whole.  An ordered compaction writes the m items of each side, in
+//      side is taken whole; each CTA's own counts below and at the cut come from its
+//      own histograms.  An ordered compaction writes the m items of each side, in
 //      position order, to keys1/idx1 (orphans at [0, m), donors at [N/2, N/2 + m)).
-//   C. Each CTA sorts its share of both lists (at most kChunk items per side) by
-//      (key, position) with a bitonic network in shared memory; an item's place in the
-//      swap list is its rank in its own share plus, for every other share, the number
-//      of that share's items ordered before it (binary search in the other CTA's
-//      shared memory).  Larger lists are sorted by one CTA per side with the stable
-//      radix passes over the workspace.
+//   C. Each CTA sorts its share of both lists by (key, position) with a bitonic
+//      network held in registers (eight slots per thread; warp shuffles for strides up
+//      to 128, shared memory beyond): both sides at once for shares of up to kChunk
+//      items, one side after the other for shares of up to 2 kChunk.  An item's place
+//      in the swap list is its rank in its own share plus, for every other share, the
+//      number of that share's items ordered before it (binary search in the other
+//      CTA's shared memory).  Larger shares are sorted by one CTA per side with the
+//      stable radix passes over the workspace.
 // Every CTA of a cluster runs the same sequence of cluster barriers: each branch and
 // loop bound that leads to one depends only on values that are identical in every CTA.
 namespace cg = cooperative_groups;
 
-constexpr int kChunk = 2048;   // items per side a CTA sorts in shared memory
+constexpr int kChunk = 2048;   // items per side a CTA sorts at once (both sides)
 
 template <int C>
 __device__ __forceinline__ void cluster_sync()
