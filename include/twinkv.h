@@ -62,8 +62,10 @@
  *
  * Precision.  The twin of each key is the argmax of fp32 tensor-core similarities
  * (bf16 products, fp32 accumulation), the lowest position on a tie; candidates within
- * about 8e-6 in similarity of the maximum count as tied, so such a near tie can go to
- * a lower position than the exact argmax.  The reported b of that twin is then
+ * about 8e-6 in similarity of the maximum (for a key of its unit's largest norm, more
+ * for smaller keys in proportion) count as tied, within each 32-column chunk at
+ * d = 128 and across all columns at d = 64, so such a near tie can go to a lower
+ * position than the exact argmax.  The reported b of that twin is then
  * recomputed as
  * (k_i . k_j) / sqrt((k_i . k_i)(k_j . k_j)) with double-float dot products (relative
  * error ~1e-13) and fp64 rounding, so it is symmetric in (i, j) and exactly 1 for a
