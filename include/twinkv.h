@@ -51,6 +51,13 @@
  * are kept until the process exits.  cudaDeviceReset on a device after the library
  * has been called there is not supported: the recorded addresses would be stale.
  *
+ * CUDA graphs.  Once a first call has run on a device outside stream capture, the
+ * device-side calls (all but twinkv_repair_host) may be captured in a CUDA graph: they
+ * only enqueue kernels and memsets on the given stream, and whatever depends on the
+ * data (retained counts, the split of the work, the selection's cut) is computed on the
+ * device, so a replay computes on the buffers' contents at replay time.  The captured
+ * pointers (inputs, outputs, workspace) must stay valid for the graph's lifetime.
+ *
  * Errors.  Argument errors that the host can see (null pointers, sizes, d, dtype,
  * window, threshold, a too-small workspace) are returned at once and nothing is
  * enqueued.  Per-unit data errors are found on the device and reported in
