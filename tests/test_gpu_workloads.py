@@ -101,7 +101,7 @@ def full_units(keys, S0, h, units, tau):
 
 
 # rows sampled per unit (the long workload samples 4096 rows of each of its 8 units)
-ROWS = {"llama": 256, "qwen": 128, "retrieval": 96, "long": 4096}
+ROWS = {"llama": 256, "qwen": 128, "retrieval": 96, "long": 4096, "largest": 256}
 
 
 def check_config(name, w, ratio, keys, truths, S0, h, full, schedule="uniform",
@@ -162,6 +162,17 @@ def test_long_full_sampled_rows():
     w = synth.get("long")
     keys, truths, S0, h = run_full(w, 0.5)
     check_config("long", w, 0.5, keys, truths, S0, h, [], seed=5)
+
+
+def test_repair_at_the_largest_n():
+    """N = 2^20, the largest the ABI accepts, on the long-stress recipe (2 heads,
+    d = 128; the selection runs each unit on a cluster of 16 CTAs): the split check and
+    the invariants on every position, every planted twin exact, and 256 random rows of
+    each unit against the oracle over all 2^20 columns."""
+    w = synth.get("long", H=2, N=1 << 20)
+    keys, truths, S0, h = run_full(w, 0.5)
+    assert int(h["nswaps"].min()) > 0
+    check_config("largest", w, 0.5, keys, truths, S0, h, [], seed=6)
 
 
 @pytest.mark.parametrize("name", ["qwen", "llama"])
