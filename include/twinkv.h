@@ -72,7 +72,10 @@
  * about 8e-6 in similarity of the maximum (for a key of its unit's largest norm, more
  * for smaller keys in proportion) count as tied, within each 32-column chunk at
  * d = 128 and across all columns at d = 64, so such a near tie can go to a lower
- * position than the exact argmax.  The reported b of that twin is then
+ * position than the exact argmax.  The band is about 2^-17 * max||k|| / ||k_i|| in
+ * similarity (max over the key's unit): keys down to 1/100 of their unit's longest
+ * stay well inside a 2e-3 tolerance; at d = 64, keys 1000 times shorter than an outlier
+ * key of their unit measured deviations up to 8e-3.  The reported b of that twin is then
  * recomputed as
  * (k_i . k_j) / sqrt((k_i . k_i)(k_j . k_j)) with double-float dot products (relative
  * error ~1e-13) and fp64 rounding, so it is symmetric in (i, j) and exactly 1 for a

@@ -366,6 +366,26 @@ def test_repair_select_every_cluster_size(cluster, N, K, tau, monkeypatch):
     split_check(h, S0, tau, 4, 64)
 
 
+@pytest.mark.parametrize("d", [128, 64])
+def test_keys_far_below_their_units_largest_norm(d):
+    """The audit's packed resolution is relative to the unit's largest key norm: a key
+    of norm ratio r to it has a near-tie band of about 2^-17 / r in similarity.  Down to
+    r = 1/100 that band stays inside the 2e-3 tolerance: every key of these units is
+    about 100 times shorter than one outlier key, with planted near-duplicates, and all
+    compare with the oracle."""
+    U, N = 2, 1500
+    rng = np.random.default_rng(d)
+    x = rng.standard_normal((U, N, d), dtype=np.float32)
+    for u in range(U):
+        src = rng.choice(N, 60, replace=False)
+        dst = (src + rng.integers(40, 400, 60)) % N
+        x[u, dst] = x[u, src] + np.float32(0.02) * rng.standard_normal((60, d), dtype=np.float32)
+        x[u, 700] *= np.float32(100.0)          # the outlier sets the unit's scale
+    rep, s, t = redundancy_vs_oracle(x, 1, U, 32)
+    assert rep.n_fail == 0, rep.notes
+    assert rep.max_dev_same_twin < 1e-9
+
+
 def test_wait_probe_times_out_cleanly():
     assert tk.twinkv_wait_probe(2_000_000) == tk.ERR_TIMEOUT
     # the context stays usable and the sticky error word is untouched
